@@ -1,0 +1,456 @@
+#!/usr/bin/env python
+"""Throughput benchmark of the GB300 CoverPrune hot path.
+
+Workload (one step): a batch of 32 independent long-video scenes (N=8192
+tokens of D=3584 bf16 features, 32 frames x 256 tokens, Zipf-sized modes,
+random-walk camera), full CoverPrune at 15% retention (K=1229): FST cost,
+FST capacity and dense SGS (every token's neighbourhood is the whole scene),
+then the kept indices.  The metric is scenes per second (whole job, all
+GPUs; each rank prunes its own 32 scenes -- weak scaling, no collective on
+the data path).  The same line reports the single-scene pruning latency,
+CoverPrune-Lite on the same batch, the dominant kernel's roofline, an
+end-to-end number through host buffers and the CPU oracle as a baseline.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With --impl reference the CPU oracle (fp64, scalar C) is timed on the host's
+cores on a bounded sample of the same workload, scaled to scenes per second.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "scenes/sec & pruning latency (N=8192,D=3584,15% keep); % HBM / tensor roofline"
+WORKLOAD = "batch32_long_video_full_sgs_15pct"
+SCENES, RETENTION = 32, 0.15
+SCENE_NAME = "long_video"
+STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output")
+
+
+def _gen(seed):
+    """Worker: one scene as bf16 bit patterns (spawned before any CUDA use)."""
+    from paper_2608_13226_gb300 import scenes
+    s = scenes.make_scene(SCENE_NAME, seed)
+    return scenes.bf16_bits(s["feats"]), s["pos"], s["frame"]
+
+
+def make_batch(seeds):
+    procs = max(1, min(len(seeds), (os.cpu_count() or 2) // 2, 16))
+    with mp.get_context("spawn").Pool(procs) as pool:
+        return pool.map(_gen, seeds)
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return d["hbm_gbs"], d["bf16_tflops"], d.get("bf16_tflops_sustained"), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# --------------------------------------------------------------------------
+# clocks under load
+# --------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.index), "-lms", "200", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self) -> dict:
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        except OSError:
+            pass
+        finally:
+            try:
+                os.unlink(self.path)
+            except OSError:
+                pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        pw = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "power_w_max": max(pw) if pw else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle: bounded sample of one scene, scaled to scenes/s
+# --------------------------------------------------------------------------
+def oracle_scene_seconds(scene, K: int) -> tuple[float, dict]:
+    """Time the CPU oracle on a bounded sample of one scene of the workload
+    and scale each stage to the whole scene by its operation count."""
+    import numpy as np
+
+    import oracle as orc
+    F = scene["feats"].astype(np.float64)
+    X, tau = scene["pos"], scene["frame"]
+    N = F.shape[0]
+    w = orc.Weights()
+    parts = {}
+    n_sub = 2048  # normalisers over the first n_sub tokens: (N / n_sub)^2 of the pairs
+    t = time.perf_counter()
+    orc.normalisers(F[:n_sub], X[:n_sub], tau[:n_sub])
+    parts["normalisers"] = (time.perf_counter() - t) * (N / n_sub) ** 2
+    nm = orc.normalisers(F[:2], X[:2], tau[:2])  # any normalisers time the same
+    rows = 512  # cost rows 0..rows of N
+    t = time.perf_counter()
+    C0 = orc.cost_rows(F, X, tau, w, nm, 0, rows)
+    parts["cost"] = (time.perf_counter() - t) * N / rows
+    t = time.perf_counter()
+    nbr = orc.knn_others(X, 8)
+    _, v = orc.capacity(F, X, tau, w, nm, 8, nbr)
+    parts["capacity"] = time.perf_counter() - t
+    steps = 24  # greedy steps on a full N x N matrix (the sweep does not depend on the values)
+    Cfull = np.tile(C0, (N // rows, 1))
+    t = time.perf_counter()
+    orc.sgs(Cfull, v, steps, 3.0)
+    parts["sgs"] = (time.perf_counter() - t) * K / steps
+    del Cfull
+    total = sum(parts.values())
+    sample = (f"one {SCENE_NAME} scene (N={N}, D={F.shape[1]}, K={K}): normalisers on "
+              f"{n_sub} tokens x{(N / n_sub) ** 2:.0f}, cost rows 0..{rows} x{N // rows}, "
+              f"full neighbours+capacity, {steps} of {K} greedy steps x{K / steps:.1f}")
+    return total, {"parts_s": {k: round(v_, 3) for k, v_ in parts.items()}, "sample": sample}
+
+
+def cpu_baseline_line(scene, K):
+    import oracle as orc
+    orc.build()
+    secs, info = oracle_scene_seconds(scene, K)
+    return {"value": 1.0 / secs, "unit": "scenes/s", "cores": orc.get_threads(),
+            "kind": "oracle", "sample": info["sample"], "scene_s": round(secs, 3),
+            "parts_s": info["parts_s"]}
+
+
+# --------------------------------------------------------------------------
+# reference arm: the oracle timed as it stands
+# --------------------------------------------------------------------------
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    from paper_2608_13226_gb300 import scenes
+    s = scenes.make_scene(SCENE_NAME, 0)
+    K = math.ceil(RETENTION * s["cfg"].N - 1e-9)
+    import oracle as orc
+    orc.build()
+    times = []
+    info = None
+    for i in range(args.warmup + args.steps):
+        secs, info = oracle_scene_seconds(s, K)
+        if i >= args.warmup:
+            times.append(secs)
+    scene_s = statistics.mean(times)
+    value = 1.0 / scene_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "scenes/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": scene_s * SCENES * 1000.0, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "scenes": SCENES, "N": s["cfg"].N,
+                       "D": s["cfg"].D, "K": K, "g": "N (dense)",
+                       "note": "each step times the oracle on a bounded sample of one scene; "
+                               "ms_per_step scales it to the 32-scene step"},
+            "cpu_baseline": {"value": value, "unit": "scenes/s", "cores": orc.get_threads(),
+                             "kind": "oracle", "sample": info["sample"]},
+            "e2e": {"value": value, "unit": "scenes/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------
+# our arm
+# --------------------------------------------------------------------------
+def run_ours(args, rank, world, local_rank, raw):
+    import numpy as np
+    import torch
+
+    import paper_2608_13226_gb300 as cp
+    from paper_2608_13226_gb300 import build as cuda_build
+    cuda_build.build()
+    cp.load()
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    N, D = 8192, 3584
+    K = cp.coverprune_budget(RETENTION, N)
+    bits = np.stack([r[0] for r in raw])
+    pos_h = np.stack([r[1] for r in raw])
+    fr_h = np.stack([r[2] for r in raw])
+    B = bits.shape[0]
+    feats_pin = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).pin_memory()
+    pos_pin = torch.from_numpy(pos_h).pin_memory()
+    fr_pin = torch.from_numpy(fr_h).pin_memory()
+    feats = feats_pin.to(dev)
+    pos = pos_pin.to(dev)
+    fr = fr_pin.to(dev)
+    prm = cp.Params()
+    stream = torch.cuda.current_stream()
+
+    ws = cp.workspace(cp.CP_OP_SELECT, B, N, D, K, cp.CP_BF16, prm, dev)
+    out = {"kept": torch.empty(B, K, dtype=torch.int64, device=dev),
+           "objective": torch.empty(B, dtype=torch.float64, device=dev)}
+
+    def step():
+        cp.coverprune_select(feats, pos, fr, K, prm, order=False, gains=False, ws=ws, out=out)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    cp.coverprune_profile_read()  # clear
+    cp.coverprune_profile_enable(True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local_rank) as clk:
+        barrier()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            step()
+        ev1.record(stream)
+        barrier()
+    cp.coverprune_profile_enable(False)
+    prof = cp.coverprune_profile_read()
+    clocks = clk.summary()
+    st = cp.coverprune_check(ws)
+    if st != cp.CP_OK:
+        raise RuntimeError(f"device status after the timed region: {cp.status_string(st)}")
+    ms_step = max_over_ranks(ev0.elapsed_time(ev1) / args.steps)
+    value = B * world / (ms_step / 1000.0)
+
+    # roofline of the dominant kernel (dense SGS sweep) from its own events
+    hbm, tf_burst, tf_sust, peak_kind = measured_peaks()
+    sgs_ms, sgs_launches = prof["sgs"]
+    sgs_bytes_per_step = B * K * (N * N * 4 + N * 4)  # C read once per greedy step + row update
+    sgs_launch_ms = sgs_ms / max(sgs_launches, 1)
+    launches_per_step = max(sgs_launches // args.steps, 1)
+    sgs_gbs = (sgs_bytes_per_step / launches_per_step) / (sgs_launch_ms / 1000.0) / 1e9
+    traffic = read_traffic("sgs")
+    roofline = {"bound": "hbm", "kernel": "k_sgs<dense>", "achieved": round(sgs_gbs, 1),
+                "peak": hbm, "unit": "GB/s", "frac": round(sgs_gbs / hbm, 4),
+                "traffic": traffic, "peak_source": peak_kind,
+                "algorithmic_bytes_per_launch": sgs_bytes_per_step // launches_per_step,
+                "avg_launch_ms": round(sgs_launch_ms, 3)}
+    def tflops(stage, flops_per_call):
+        ms, launches = prof[stage]
+        if ms <= 0 or launches <= 0:
+            return None
+        per_launch = flops_per_call * args.steps / launches
+        return per_launch / (ms / launches / 1000.0) / 1e12
+
+    cost_tf = tflops("cost", B * 2.0 * N * N * D)            # full N x N x D product
+    gram_tf = tflops("gram", B * 1.0 * N * (N + 1) * D)      # the pairs i <= j once
+    roofline_gemm = {"bound": "tensor", "unit": "TFLOP/s", "peak": tf_burst,
+                     "cost_gemm": {"achieved": cost_tf and round(cost_tf, 1),
+                                   "frac": cost_tf and round(cost_tf / tf_burst, 4),
+                                   "flops_per_launch": B * 2 * N * N * D},
+                     "normaliser_gemm": {"achieved": gram_tf and round(gram_tf, 1),
+                                         "frac": gram_tf and round(gram_tf / tf_burst, 4),
+                                         "flops_per_launch": B * N * (N + 1) * D},
+                     "peak_source": peak_kind}
+    stages = {k: round(v[0] / args.steps, 3) for k, v in prof.items() if v[0] > 0}
+    gpu_launches = sum(v[1] for v in prof.values())
+
+    # single-scene pruning latency
+    ws1 = cp.workspace(cp.CP_OP_SELECT, 1, N, D, K, cp.CP_BF16, prm, dev)
+    lat = []
+    for i in range(6):
+        barrier()
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        cp.coverprune_select(feats[0], pos[0], fr[0], K, prm, order=False, gains=False, ws=ws1)
+        b_.record(stream)
+        torch.cuda.synchronize()
+        if i >= 2:
+            lat.append(a.elapsed_time(b_))
+    latency_ms = statistics.median(lat)
+    del ws1
+
+    # CoverPrune-Lite on the same batch
+    wsl = cp.workspace(cp.CP_OP_LITE, B, N, D, K, cp.CP_BF16, prm, dev)
+    lite_out = {"kept": torch.empty(B, K, dtype=torch.int64, device=dev)}
+    for _ in range(args.warmup):
+        cp.coverprune_lite_select(feats, pos, fr, K, prm, group_start=False, objective=False,
+                                  ws=wsl, out=lite_out)
+    barrier()
+    cp.coverprune_profile_read()
+    cp.coverprune_profile_enable(True)
+    a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        cp.coverprune_lite_select(feats, pos, fr, K, prm, group_start=False, objective=False,
+                                  ws=wsl, out=lite_out)
+    b_.record(stream)
+    barrier()
+    cp.coverprune_profile_enable(False)
+    lprof = cp.coverprune_profile_read()
+    lite_ms = max_over_ranks(a.elapsed_time(b_) / args.steps)
+    lat_l = []
+    for i in range(6):
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        cp.coverprune_lite_select(feats[0], pos[0], fr[0], K, prm, group_start=False,
+                                  objective=False)
+        b_.record(stream)
+        torch.cuda.synchronize()
+        if i >= 2:
+            lat_l.append(a.elapsed_time(b_))
+    lite = {"scenes_per_s": B * world / (lite_ms / 1000.0), "ms_per_step": round(lite_ms, 3),
+            "latency_ms": round(statistics.median(lat_l), 3),
+            "stages_ms": {k: round(v[0] / args.steps, 3) for k, v in lprof.items() if v[0] > 0}}
+    del wsl
+
+    # end to end through the C ABI with host buffers: H2D of the step's inputs
+    # from pinned memory, the call, D2H of the kept indices and objectives
+    kept_pin = torch.empty(B, K, dtype=torch.int64).pin_memory()
+    obj_pin = torch.empty(B, dtype=torch.float64).pin_memory()
+    f_dev = torch.empty_like(feats)
+    p_dev = torch.empty_like(pos)
+    t_dev = torch.empty_like(fr)
+
+    def e2e_step():
+        f_dev.copy_(feats_pin, non_blocking=True)
+        p_dev.copy_(pos_pin, non_blocking=True)
+        t_dev.copy_(fr_pin, non_blocking=True)
+        cp.coverprune_select(f_dev, p_dev, t_dev, K, prm, order=False, gains=False, ws=ws,
+                             out=out)
+        kept_pin.copy_(out["kept"], non_blocking=True)
+        obj_pin.copy_(out["objective"], non_blocking=True)
+
+    e2e_step()
+    barrier()
+    a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(max(2, args.steps // 2)):
+        e2e_step()
+    b_.record(stream)
+    barrier()
+    e2e_ms = max_over_ranks(a.elapsed_time(b_) / max(2, args.steps // 2))
+    h2d = feats_pin.numel() * 2 + pos_pin.numel() * 4 + fr_pin.numel() * 4
+    d2h = kept_pin.numel() * 8 + obj_pin.numel() * 8
+    e2e = {"value": B * world / (e2e_ms / 1000.0), "unit": "scenes/s",
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 3)}
+
+    if rank != 0:
+        if dist is not None:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+    cpu = None
+    if world == 1:
+        s0 = {"feats": (bits[0].astype(np.uint32) << 16).view(np.float32), "pos": pos_h[0],
+              "frame": fr_h[0]}
+        cpu = cpu_baseline_line(s0, K)
+    line = {"metric": METRIC, "value": value, "unit": "scenes/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "scenes_per_gpu": B, "N": N, "D": D, "K": K,
+                       "retention": RETENTION, "g": "N (dense)", "input_dtype": "bf16",
+                       "l2": "inputs larger than L2 (1.9 GB features, 8.6 GB cost per step)",
+                       "generator": "paper_2608_13226_gb300.scenes long_video, seeds "
+                                    f"{rank * B}..{rank * B + B - 1} per rank"},
+            "latency_ms": round(latency_ms, 3),
+            "lite": lite, "roofline": roofline, "roofline_gemm": roofline_gemm,
+            "stages_ms": stages, "gpu_launches": gpu_launches, "e2e": e2e,
+            "clocks": clocks, "cpu_baseline": cpu}
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def read_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary of this kernel,
+    if one exists for the current build (a line 'traffic_bytes_per_launch: X')."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
+    try:
+        for line in open(path):
+            if line.startswith("traffic_bytes_per_launch:"):
+                v = line.split(":", 1)[1].strip()
+                return None if v in ("", "null") else float(v)
+    except OSError:
+        pass
+    return None
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    # scenes are drawn in a spawned pool before any CUDA use
+    raw = make_batch(list(range(rank * SCENES, rank * SCENES + SCENES)))
+    run_ours(args, rank, world, local_rank, raw)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,139 @@
+// Internal declarations of the CoverPrune CUDA library: parameter blocks
+// passed to kernels, per-scene normalisers and the host-side launchers of
+// every kernel.  Not part of the public ABI (include/coverprune.h is).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/coverprune.h"
+
+namespace cp {
+
+// Method parameters in the form the kernels use them.
+struct DevParams {
+  float lambda_f, lambda_x, lambda_tau;
+  float kappa, inv_log1p_kappa;
+  float alpha_f, alpha_x, alpha_tau;
+  float voxel, m0;
+  int n_cap;   // capacity neighbours, already clamped to N-1
+  int g;       // SGS neighbourhood incl. the token itself; == N means all
+  int kk;      // neighbours stored per token = max(n_cap, g-1) (g < N) or n_cap
+  int cap_mode;
+  uint64_t timeout_ns;
+};
+
+// Per-scene min-max normalisers (Sec. 3.3).  lo/hi are the extremes of each
+// discrepancy; *_rinv = 1 / (hi - lo), or 0 when the range is <= 1e-6 (the
+// normalised term is then 0).
+struct SceneNorms {
+  float f_lo, f_hi, x_lo, x_hi, t_lo, t_hi;
+  float f_rinv, x_rinv, t_rinv;
+  float pad[7];
+};
+static_assert(sizeof(SceneNorms) == 64, "SceneNorms layout");
+
+// Raw per-scene statistics gathered by atomics before the normalisers are
+// finalised: order-preserving keys of max/min cosine and max squared
+// distance, frame range and the bounding-box minimum (Morton origin).
+struct SceneStats {
+  uint32_t cos_max_key, cos_min_key, d2_max_bits;
+  int32_t tau_min, tau_max;
+  float bbox_min[3];
+  uint32_t pad[8];
+};
+static_assert(sizeof(SceneStats) == 64, "SceneStats layout");
+
+constexpr double kRangeEps = 1e-6;
+
+// Device attributes cached per device.
+struct DeviceInfo {
+  int sm_count;
+  int max_smem_optin;
+  int cc_major, cc_minor;
+};
+int device_info(DeviceInfo* out);
+
+// ---------------------------------------------------------------------------
+// Launchers (each returns a cp_status; all enqueue on `s`).
+// ---------------------------------------------------------------------------
+
+// K0: per-scene frame range and bounding-box minimum; initialises the
+// atomically reduced fields of `stats`.
+int launch_scene_stats(const float* pos, const int32_t* frame, int64_t B, int64_t N,
+                       SceneStats* stats, cudaStream_t s);
+// K0: inverse feature norms inv[b*N + j] (0 for a zero feature).
+int launch_inv_norms(const void* feats, int dtype, int64_t B, int64_t N, int64_t D,
+                     float* inv, cudaStream_t s);
+// K1: per token the kk nearest other tokens by (fp32 d^2, index) into
+// nbr[(b*N + j)*kk + q]; also the scene's largest squared distance.
+int launch_knn(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
+               cudaStream_t s);
+// K2 (fp32 SIMT and bf16 tensor-core variants): max and min cosine over all
+// pairs into stats.
+int launch_gram_minmax(const void* feats, int dtype, const float* inv, int64_t B, int64_t N,
+                       int64_t D, SceneStats* stats, int* status, uint64_t timeout_ns,
+                       cudaStream_t s);
+// Scene diameter sqrt(max d^2) from stats into out[b].
+int launch_diameter(const SceneStats* stats, int64_t B, float* out, cudaStream_t s);
+// Normalisers from stats.  Optionally also the public [B, 6] float copy.
+int launch_finalize_norms(const SceneStats* stats, int64_t B, SceneNorms* norms,
+                          float* norms_out, cudaStream_t s);
+// K3: the FST cost C[b][s][t] into cost + b*N*ldc + s*ldc + t for t < N;
+// columns N <= t < ldc are written as 0.
+int launch_cost(const void* feats, int dtype, const float* inv, const float* pos,
+                const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
+                int64_t N, int64_t D, float* cost, int64_t ldc, int* status, cudaStream_t s);
+// K4: capacity score r and capacity v (Eqs. fst_capacity_score, fst_capacity).
+int launch_capacity(const void* feats, int dtype, const float* inv, const float* pos,
+                    const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
+                    const DevParams& P, int64_t B, int64_t N, int64_t D, float* r, float* v,
+                    float* v_out, cudaStream_t s);
+// Local SGS: slab[b][t][k] = C(t, M_g(t)[k]) gathered from the dense cost.
+int launch_slab(const float* cost, int64_t ldc, const int32_t* nbr, const DevParams& P,
+                int64_t B, int64_t N, float* slab, cudaStream_t s);
+// K5: K greedy steps; order32[b*K + l] = token added at step l.
+int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
+               const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
+               int32_t* order32, float* gains, double* objective, uint64_t* partials,
+               uint32_t* counters, int* status, cudaStream_t s);
+// Sort the B rows of K int32 indices ascending into int64 (and copy the
+// unsorted order out as int64 if order64 != NULL).
+int launch_sort_kept(const int32_t* idx32, int64_t B, int64_t K, int64_t* kept,
+                     int64_t* order64, cudaStream_t s);
+// K6: Morton order perm[b*N + p].
+int launch_morton(const float* pos, const SceneStats* stats, const DevParams& P, int64_t B,
+                  int64_t N, int32_t* perm, cudaStream_t s);
+// K7: capacity-guided group starts gs[b*(K+1) + q] (int32).
+int launch_groups(const float* v, const int32_t* perm, int64_t B, int64_t N, int64_t K,
+                  uint64_t* prefix, int32_t* gs, cudaStream_t s);
+// K8: per-group prototype and its score; objective = sum of scores.
+int launch_lite_proto(const void* feats, int dtype, const float* inv, const float* pos,
+                      const int32_t* frame, const SceneNorms* norms, const float* v,
+                      const int32_t* perm, const int32_t* gs, const DevParams& P, int64_t B,
+                      int64_t N, int64_t D, int64_t K, int32_t* proto, double* score,
+                      double* objective, cudaStream_t s);
+// K9: row gather of the kept tokens.
+int launch_gather(const void* feats, int dtype, const float* pos, const int32_t* frame,
+                  int64_t B, int64_t N, int64_t D, const int64_t* kept, int64_t K,
+                  void* feats_out, float* pos_out, int32_t* frame_out, int32_t* status,
+                  cudaStream_t s);
+// Barrier self-test (see coverprune_barrier_selftest).
+int launch_barrier_selftest(int n_blocks, int expected, uint64_t timeout_ns, uint32_t* ctr,
+                            int* status, cudaStream_t s);
+
+// Largest N the selection kernels keep in shared memory.
+constexpr int64_t kMaxSelectN = 16384;
+// Largest N whose neighbour keys fit one block's shared memory.
+constexpr int64_t kMaxKnnN = 49152;
+
+// Counts one kernel launch under the calling thread's current stage.
+void note_launch();
+inline int cuda_status(cudaError_t e) { return e == cudaSuccess ? CP_OK : CP_ECUDA; }
+// After every <<<>>> launch: count it and report launch errors.
+inline int last_launch_status() {
+  note_launch();
+  return cuda_status(cudaGetLastError());
+}
+
+}  // namespace cp

@@ -1,0 +1,284 @@
+// K0 (scene statistics, inverse feature norms), K1 (3D nearest neighbours and
+// scene diameter) and the min-max normalisers of Sec. 3.3.
+#include "common.cuh"
+
+namespace cp {
+
+// ---------------------------------------------------------------------------
+// K0a: frame range (0 when frame is NULL) and bounding-box minimum per scene;
+// initialises the fields that later kernels reduce into atomically.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(512) k_scene_stats(const float* __restrict__ pos,
+                                                     const int32_t* __restrict__ frame,
+                                                     int N, SceneStats* stats) {
+  const int b = blockIdx.x;
+  const float* X = pos + (size_t)b * N * 3;
+  const int32_t* T = frame ? frame + (size_t)b * N : nullptr;  // may be absent
+  int tmin = INT32_MAX, tmax = INT32_MIN;
+  float lo[3] = {INFINITY, INFINITY, INFINITY};
+  for (int j = threadIdx.x; j < N; j += blockDim.x) {
+    const int t = T ? T[j] : 0;
+    tmin = min(tmin, t);
+    tmax = max(tmax, t);
+#pragma unroll
+    for (int a = 0; a < 3; ++a) lo[a] = fminf(lo[a], X[3 * j + a]);
+  }
+  __shared__ int s_tmin[16], s_tmax[16];
+  __shared__ float s_lo[3][16];
+  for (int o = 16; o > 0; o >>= 1) {
+    tmin = min(tmin, __shfl_xor_sync(0xFFFFFFFFu, tmin, o));
+    tmax = max(tmax, __shfl_xor_sync(0xFFFFFFFFu, tmax, o));
+#pragma unroll
+    for (int a = 0; a < 3; ++a) lo[a] = fminf(lo[a], __shfl_xor_sync(0xFFFFFFFFu, lo[a], o));
+  }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  if (l == 0) {
+    s_tmin[w] = tmin;
+    s_tmax[w] = tmax;
+    for (int a = 0; a < 3; ++a) s_lo[a][w] = lo[a];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int nw = blockDim.x >> 5;
+    for (int i = 1; i < nw; ++i) {
+      tmin = min(tmin, s_tmin[i]);
+      tmax = max(tmax, s_tmax[i]);
+      for (int a = 0; a < 3; ++a) lo[a] = fminf(lo[a], s_lo[a][i]);
+    }
+    SceneStats st;
+    st.cos_max_key = 0u;           // below every real key
+    st.cos_min_key = 0xFFFFFFFFu;  // above every real key
+    st.d2_max_bits = 0u;           // d^2 >= 0: float bits order like the values
+    st.tau_min = tmin;
+    st.tau_max = tmax;
+    for (int a = 0; a < 3; ++a) st.bbox_min[a] = lo[a];
+    for (int i = 0; i < 8; ++i) st.pad[i] = 0u;
+    stats[b] = st;
+  }
+}
+
+int launch_scene_stats(const float* pos, const int32_t* frame, int64_t B, int64_t N,
+                       SceneStats* stats, cudaStream_t s) {
+  k_scene_stats<<<(unsigned)B, 512, 0, s>>>(pos, frame, (int)N, stats);
+  return last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// K0b: inv[j] = 1 / ||f_j|| (0 for a zero feature), one warp per token.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ F, int64_t rows, int D,
+                                                   float* __restrict__ inv) {
+  const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const T* f = F + row * D;
+  constexpr int V = Vec16<T>::n;
+  float acc = 0.0f;
+  for (int d = lane * V; d < D; d += 32 * V) {
+    float x[V];
+    Vec16<T>::load(f + d, x);
+#pragma unroll
+    for (int i = 0; i < V; ++i) acc = fmaf(x[i], x[i], acc);
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) inv[row] = acc > 0.0f ? 1.0f / sqrtf(acc) : 0.0f;
+}
+
+int launch_inv_norms(const void* feats, int dtype, int64_t B, int64_t N, int64_t D, float* inv,
+                     cudaStream_t s) {
+  const int64_t rows = B * N;
+  const unsigned grid = (unsigned)((rows + 7) / 8);
+  if (dtype == CP_BF16)
+    k_inv_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)feats, rows, (int)D, inv);
+  else
+    k_inv_norms<float><<<grid, 256, 0, s>>>((const float*)feats, rows, (int)D, inv);
+  return last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// K1: for token j, its kk nearest other tokens ordered by (fp32 d^2, index)
+// (capacity set N_n of Eq. fst_capacity_score and SGS neighbourhood M_g of
+// Eq. local_neighbor), and the largest squared distance of the row (for the
+// spatial normaliser).  One block per token; the N keys live in shared
+// memory; the kk-th smallest key is found by bisection on its bit pattern
+// (d^2 >= 0, so float bits order like the values), the winners are collected
+// in index order and sorted by (key, index).
+// ---------------------------------------------------------------------------
+constexpr int KNN_THREADS = 256;
+
+__device__ __forceinline__ int block_sum_int(int v, int* s_red) {
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) s_red[w] = v;
+  __syncthreads();
+  int t = 0;
+  for (int i = 0; i < KNN_THREADS / 32; ++i) t += s_red[i];
+  return t;
+}
+
+__global__ void __launch_bounds__(KNN_THREADS) k_knn(const float* __restrict__ pos, int N, int kk,
+                                                     int list_len, int32_t* __restrict__ nbr,
+                                                     SceneStats* stats) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  unsigned long long* list = reinterpret_cast<unsigned long long*>(smem);  // [list_len]
+  uint32_t* key = reinterpret_cast<uint32_t*>(list + list_len);            // [N]
+  __shared__ int s_red[KNN_THREADS / 32];
+  __shared__ uint32_t s_redu[KNN_THREADS / 32];
+  __shared__ int s_wcnt[2][KNN_THREADS / 32];
+
+  const int j = blockIdx.x, b = blockIdx.y;
+  const float* X = pos + (size_t)b * N * 3;
+  const float xj = X[3 * j], yj = X[3 * j + 1], zj = X[3 * j + 2];
+  uint32_t dmax = 0u;
+  for (int k = threadIdx.x; k < N; k += KNN_THREADS) {
+    float d2 = sqdist_rn(xj, yj, zj, X[3 * k], X[3 * k + 1], X[3 * k + 2]);
+    uint32_t bits = __float_as_uint(d2);
+    dmax = max(dmax, bits);
+    key[k] = (k == j) ? 0xFFFFFFFFu : bits;
+  }
+  for (int o = 16; o > 0; o >>= 1) dmax = max(dmax, __shfl_xor_sync(0xFFFFFFFFu, dmax, o));
+  if ((threadIdx.x & 31) == 0) s_redu[threadIdx.x >> 5] = dmax;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < KNN_THREADS / 32; ++i) dmax = max(dmax, s_redu[i]);
+    atomicMax(&stats[b].d2_max_bits, dmax);
+  }
+  if (kk <= 0) return;
+
+  // bisection: smallest T with #{key <= T} >= kk
+  uint32_t lo = 0u, hi = 0xFFFFFFFEu;
+  while (lo < hi) {
+    const uint32_t mid = lo + ((hi - lo) >> 1);
+    int c = 0;
+    for (int k = threadIdx.x; k < N; k += KNN_THREADS) c += key[k] <= mid;
+    c = block_sum_int(c, s_red);
+    if (c >= kk) hi = mid; else lo = mid + 1;
+  }
+  const uint32_t T = lo;
+  int less = 0;
+  for (int k = threadIdx.x; k < N; k += KNN_THREADS) less += key[k] < T;
+  less = block_sum_int(less, s_red);
+  const int need_eq = kk - less;
+
+  // collect in index order: every key < T, and the first need_eq keys == T
+  for (int i = threadIdx.x; i < list_len; i += KNN_THREADS) list[i] = ~0ull;
+  __syncthreads();
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  int base = 0, eq_taken = 0;
+  for (int c0 = 0; c0 < N; c0 += KNN_THREADS) {
+    const int k = c0 + threadIdx.x;
+    const uint32_t kv = k < N ? key[k] : 0xFFFFFFFFu;
+    const bool is_eq = kv == T && k < N;
+    // rank among equal keys of this chunk, in index order
+    const unsigned beq = __ballot_sync(0xFFFFFFFFu, is_eq);
+    if (l == 0) s_wcnt[0][w] = __popc(beq);
+    __syncthreads();
+    int eq_before = 0, eq_total = 0;
+    for (int i = 0; i < KNN_THREADS / 32; ++i) {
+      eq_before += i < w ? s_wcnt[0][i] : 0;
+      eq_total += s_wcnt[0][i];
+    }
+    const int rank_eq = eq_taken + eq_before + __popc(beq & ((1u << l) - 1u));
+    const bool take = (kv < T && k < N) || (is_eq && rank_eq < need_eq);
+    const unsigned bt = __ballot_sync(0xFFFFFFFFu, take);
+    if (l == 0) s_wcnt[1][w] = __popc(bt);
+    __syncthreads();
+    int t_before = 0, t_total = 0;
+    for (int i = 0; i < KNN_THREADS / 32; ++i) {
+      t_before += i < w ? s_wcnt[1][i] : 0;
+      t_total += s_wcnt[1][i];
+    }
+    if (take) {
+      const int p = base + t_before + __popc(bt & ((1u << l) - 1u));
+      list[p] = ((unsigned long long)kv << 32) | (unsigned)k;
+    }
+    base += t_total;
+    eq_taken += eq_total;
+    __syncthreads();
+  }
+  // bitonic sort of list[0, list_len) ascending by (key, index)
+  for (int size = 2; size <= list_len; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < (list_len >> 1); i += KNN_THREADS) {
+        const int a = 2 * i - (i & (stride - 1));
+        const int c = a + stride;
+        const bool up = (a & size) == 0;
+        const unsigned long long x = list[a], y = list[c];
+        if ((x > y) == up) { list[a] = y; list[c] = x; }
+      }
+      __syncthreads();
+    }
+  }
+  int32_t* out = nbr + ((size_t)b * N + j) * kk;
+  for (int q = threadIdx.x; q < kk; q += KNN_THREADS) out[q] = (int32_t)(list[q] & 0xFFFFFFFFu);
+}
+
+int launch_knn(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
+               cudaStream_t s) {
+  int list_len = 1;
+  while (list_len < kk) list_len <<= 1;
+  if (list_len < 2) list_len = 2;
+  const size_t smem = sizeof(unsigned long long) * list_len + sizeof(uint32_t) * (size_t)N;
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (smem > 48 * 1024 && dev < 64 && !attr_set[dev]) {
+    DeviceInfo di;
+    if (device_info(&di) != CP_OK) return CP_ECUDA;
+    if (cudaFuncSetAttribute(k_knn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             di.max_smem_optin) != cudaSuccess)
+      return CP_ECUDA;
+    attr_set[dev] = true;
+  }
+  dim3 grid((unsigned)N, (unsigned)B);
+  k_knn<<<grid, KNN_THREADS, smem, s>>>(pos, (int)N, kk, list_len, nbr, stats);
+  return last_launch_status();
+}
+
+__global__ void k_diameter(const SceneStats* stats, int B, float* out) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) out[b] = sqrtf(__uint_as_float(stats[b].d2_max_bits));
+}
+
+int launch_diameter(const SceneStats* stats, int64_t B, float* out, cudaStream_t s) {
+  k_diameter<<<(unsigned)((B + 127) / 128), 128, 0, s>>>(stats, (int)B, out);
+  return last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// Normalisers from the reduced statistics.
+// ---------------------------------------------------------------------------
+__global__ void k_finalize_norms(const SceneStats* stats, int B, SceneNorms* norms,
+                                 float* norms_out) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const SceneStats st = stats[b];
+  SceneNorms nm;
+  const float cmax = key2f(st.cos_max_key), cmin = key2f(st.cos_min_key);
+  nm.f_lo = 1.0f - cmax;
+  nm.f_hi = 1.0f - cmin;
+  nm.x_lo = 0.0f;  // diagonal pairs: d_x(j, j) = 0
+  nm.x_hi = sqrtf(__uint_as_float(st.d2_max_bits));
+  nm.t_lo = 0.0f;  // d_tau(j, j) = 0 and d_tau >= 0
+  nm.t_hi = (float)(st.tau_max - st.tau_min);
+  const float rf = nm.f_hi - nm.f_lo, rx = nm.x_hi - nm.x_lo, rt = nm.t_hi - nm.t_lo;
+  nm.f_rinv = rf > (float)kRangeEps ? 1.0f / rf : 0.0f;
+  nm.x_rinv = rx > (float)kRangeEps ? 1.0f / rx : 0.0f;
+  nm.t_rinv = rt > (float)kRangeEps ? 1.0f / rt : 0.0f;
+  for (int i = 0; i < 7; ++i) nm.pad[i] = 0.0f;
+  norms[b] = nm;
+  if (norms_out) {
+    float* o = norms_out + 6 * (size_t)b;
+    o[0] = nm.f_lo; o[1] = nm.f_hi; o[2] = nm.x_lo; o[3] = nm.x_hi; o[4] = nm.t_lo; o[5] = nm.t_hi;
+  }
+}
+
+int launch_finalize_norms(const SceneStats* stats, int64_t B, SceneNorms* norms,
+                          float* norms_out, cudaStream_t s) {
+  k_finalize_norms<<<(unsigned)((B + 127) / 128), 128, 0, s>>>(stats, (int)B, norms, norms_out);
+  return last_launch_status();
+}
+
+}  // namespace cp

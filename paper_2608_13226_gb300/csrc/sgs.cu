@@ -1,0 +1,318 @@
+// K5: Spatial-Guided Greedy Selection (Sec. 3.5, Eqs. srpot, local_neighbor,
+// greedy_flow, sgs_select, sgs_update).
+//
+// The semi-relaxed OT of Eq. srpot, with the source support and its capacity
+// as decision variables, has a closed-form plan: every target t_j sends its
+// mass v_j to its cheapest selected source among those whose neighbourhood
+// M_g contains it.  Its value is F(S) = sum_j v_j m_j with the coverage cost
+// m_j = min(m0, min_{s in S, j in M_g(s)} C(s, j)), and the residual-weighted
+// marginal cost of adding t is -gain(t) with
+//     gain(t) = sum_{j in M_g(t)} v_j max(m_j - C(t, j), 0).
+// Each step adds the unselected token with the largest gain (lowest index
+// among equal gains) and lowers m on its neighbourhood.
+//
+// One persistent cooperative grid: each scene owns `cps` co-resident blocks.
+// Every block keeps the whole (m_j, v_j) state of its scene in shared memory;
+// per step the blocks sweep disjoint candidate rows (one warp per row,
+// float4 streaming loads of C), publish their best (gain, index) key, meet at
+// a scene-local grid barrier (bounded wait), all reduce the same partials to
+// the same winner and apply the same update to their copy of m.
+#include "common.cuh"
+
+namespace cp {
+
+constexpr int SGS_THREADS = 512;
+constexpr int SGS_WARPS = SGS_THREADS / 32;
+
+__device__ __forceinline__ float4 ld_stream_f4(const float4* p) {
+  float4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
+               : "l"(p));
+  return r;
+}
+
+__device__ __forceinline__ unsigned long long gain_key(float gain, int t) {
+  // gain >= 0, so its bits order like its value; lower index wins ties
+  return ((unsigned long long)__float_as_uint(gain) << 32) | (0xFFFFFFFFu - (uint32_t)t);
+}
+
+template <bool LOCAL>
+__global__ void __launch_bounds__(SGS_THREADS) k_sgs(
+    const float* __restrict__ cost, int64_t ldc, const float* __restrict__ slab,
+    const int32_t* __restrict__ nbr, const float* __restrict__ v_all, DevParams P, int N, int K,
+    int cps, int scene0, int32_t* __restrict__ order32, float* __restrict__ gains,
+    double* __restrict__ objective, unsigned long long* partials, uint32_t* counters,
+    int* status) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int ncols = LOCAL ? N : (int)ldc;  // dense rows are padded to ldc (C = 0, v = 0)
+  float* sm_m = reinterpret_cast<float*>(smem);                  // [ncols] coverage cost m_j
+  float* sm_v = sm_m + ncols;                                    // [ncols] capacity v_j
+  uint32_t* chosen = reinterpret_cast<uint32_t*>(sm_v + ncols);  // [ceil(N/32)] bitset
+  __shared__ unsigned long long s_best[SGS_WARPS];
+  __shared__ int s_pick;
+  __shared__ float s_gain;
+
+  const int b = scene0 + blockIdx.x / cps;
+  const int c = blockIdx.x % cps;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* v = v_all + (size_t)b * N;
+  const float* Cb = LOCAL ? nullptr : cost + (size_t)b * N * ldc;
+  const float* Sb = LOCAL ? slab + (size_t)b * N * P.g : nullptr;
+  const int32_t* NB = nbr + (size_t)b * N * P.kk;
+  unsigned long long* part = partials;  // [2][B][cps]
+  const int nchosen = (N + 31) >> 5;
+
+  for (int j = threadIdx.x; j < ncols; j += SGS_THREADS) {
+    sm_m[j] = j < N ? P.m0 : 0.0f;
+    sm_v[j] = j < N ? v[j] : 0.0f;
+  }
+  for (int i = threadIdx.x; i < nchosen; i += SGS_THREADS) chosen[i] = 0u;
+  __syncthreads();
+
+  const int gw = c * SGS_WARPS + w, nw = cps * SGS_WARPS;
+  const size_t nscenes = gridDim.x / cps;
+  bool alive = true;
+  for (int step = 0; step < K && alive; ++step) {
+    unsigned long long best = 0ull;
+    for (int t = gw; t < N; t += nw) {
+      if (chosen[t >> 5] & (1u << (t & 31))) continue;
+      float acc = 0.0f;
+      if (!LOCAL) {
+        const float4* row = reinterpret_cast<const float4*>(Cb + (size_t)t * ldc);
+        const float4* m4 = reinterpret_cast<const float4*>(sm_m);
+        const float4* v4 = reinterpret_cast<const float4*>(sm_v);
+        const int nq = ncols >> 2;
+        int q = lane;
+        for (; q + 96 < nq; q += 128) {
+          float4 c0 = ld_stream_f4(row + q), c1 = ld_stream_f4(row + q + 32);
+          float4 c2 = ld_stream_f4(row + q + 64), c3 = ld_stream_f4(row + q + 96);
+          const float4 cs[4] = {c0, c1, c2, c3};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const float4 mm = m4[q + 32 * u], vv = v4[q + 32 * u];
+            acc += vv.x * fmaxf(mm.x - cs[u].x, 0.0f);
+            acc += vv.y * fmaxf(mm.y - cs[u].y, 0.0f);
+            acc += vv.z * fmaxf(mm.z - cs[u].z, 0.0f);
+            acc += vv.w * fmaxf(mm.w - cs[u].w, 0.0f);
+          }
+        }
+        for (; q < nq; q += 32) {
+          const float4 c0 = ld_stream_f4(row + q);
+          const float4 mm = m4[q], vv = v4[q];
+          acc += vv.x * fmaxf(mm.x - c0.x, 0.0f);
+          acc += vv.y * fmaxf(mm.y - c0.y, 0.0f);
+          acc += vv.z * fmaxf(mm.z - c0.z, 0.0f);
+          acc += vv.w * fmaxf(mm.w - c0.w, 0.0f);
+        }
+      } else {
+        const float* srow = Sb + (size_t)t * P.g;
+        const int32_t* nb = NB + (size_t)t * P.kk;
+        for (int k = lane; k < P.g; k += 32) {
+          const int j = k == 0 ? t : nb[k - 1];
+          acc += sm_v[j] * fmaxf(sm_m[j] - srow[k], 0.0f);
+        }
+      }
+      acc = warp_sum(acc);  // identical in every lane
+      const unsigned long long key = gain_key(acc, t);
+      best = key > best ? key : best;
+    }
+    if (lane == 0) s_best[w] = best;
+    __syncthreads();
+    const int par = step & 1;
+    if (threadIdx.x == 0) {
+      unsigned long long m = s_best[0];
+      for (int i = 1; i < SGS_WARPS; ++i) m = s_best[i] > m ? s_best[i] : m;
+      part[((size_t)par * nscenes + (b - scene0)) * cps + c] = m;
+    }
+    if (!grid_barrier(counters + b, (uint32_t)(step + 1) * (uint32_t)cps, status, P.timeout_ns)) {
+      alive = false;
+      break;
+    }
+    if (w == 0) {
+      unsigned long long m = 0ull;
+      const unsigned long long* pp = part + ((size_t)par * nscenes + (b - scene0)) * cps;
+      for (int i = lane; i < cps; i += 32) {
+        const unsigned long long x = __ldcg(pp + i);
+        m = x > m ? x : m;
+      }
+      m = warp_max_u64(m);
+      if (lane == 0) {
+        s_pick = (int)(0xFFFFFFFFu - (uint32_t)(m & 0xFFFFFFFFull));
+        s_gain = __uint_as_float((uint32_t)(m >> 32));
+      }
+    }
+    __syncthreads();
+    const int pick = s_pick;
+    if (pick < 0 || pick >= N || (chosen[pick >> 5] & (1u << (pick & 31)))) {
+      if (threadIdx.x == 0) set_status(status, CP_EDEVICE);  // never expected
+      alive = false;
+      break;
+    }
+    if (threadIdx.x == 0) {
+      chosen[pick >> 5] |= 1u << (pick & 31);
+      if (c == 0) {
+        order32[(size_t)b * K + step] = pick;
+        if (gains) gains[(size_t)b * K + step] = s_gain;
+      }
+    }
+    // S <- S u {t*} (Eq. sgs_update): lower the coverage cost of its targets
+    if (!LOCAL) {
+      const float* row = Cb + (size_t)pick * ldc;
+      for (int j = threadIdx.x; j < N; j += SGS_THREADS) sm_m[j] = fminf(sm_m[j], __ldg(row + j));
+    } else {
+      const float* srow = Sb + (size_t)pick * P.g;
+      const int32_t* nb = NB + (size_t)pick * P.kk;
+      for (int k = threadIdx.x; k < P.g; k += SGS_THREADS) {
+        const int j = k == 0 ? pick : nb[k - 1];
+        sm_m[j] = fminf(sm_m[j], srow[k]);
+      }
+    }
+    __syncthreads();
+  }
+
+  if (c == 0 && alive && objective) {
+    double part_sum = 0.0;
+    for (int j = threadIdx.x; j < N; j += SGS_THREADS)
+      part_sum += (double)sm_v[j] * (double)sm_m[j];
+    part_sum = warp_sum(part_sum);
+    __shared__ double s_obj[SGS_WARPS];
+    if (lane == 0) s_obj[w] = part_sum;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      double t = 0.0;
+      for (int i = 0; i < SGS_WARPS; ++i) t += s_obj[i];
+      objective[b] = t;
+    }
+  }
+}
+
+template <bool LOCAL>
+static int sgs_launch_impl(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
+                           const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
+                           int32_t* order32, float* gains, double* objective,
+                           unsigned long long* partials, uint32_t* counters, int* status,
+                           cudaStream_t s) {
+  DeviceInfo di;
+  if (device_info(&di) != CP_OK) return CP_ECUDA;
+  const int64_t ncols = LOCAL ? N : ldc;
+  const size_t smem = 2 * sizeof(float) * (size_t)ncols + sizeof(uint32_t) * (size_t)((N + 31) / 32);
+  auto fn = k_sgs<LOCAL>;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return CP_ECUDA;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SGS_THREADS, smem) != cudaSuccess)
+    return CP_ECUDA;
+  if (per_sm < 1) return CP_EUNSUPPORTED;
+  const int64_t slots = (int64_t)per_sm * di.sm_count;
+  const int64_t per_launch = B < slots ? B : slots;  // scenes resident together
+  int cps = (int)(slots / per_launch);
+  // a scene never needs more blocks than it has candidate rows per warp
+  const int64_t max_cps = (N + SGS_WARPS - 1) / SGS_WARPS;
+  if (cps > max_cps) cps = (int)max_cps;
+  if (cps < 1) cps = 1;
+  if (cudaMemsetAsync(counters, 0, sizeof(uint32_t) * (size_t)B, s) != cudaSuccess) return CP_ECUDA;
+  if (cudaMemsetAsync(partials, 0, sizeof(unsigned long long) * 2 * (size_t)per_launch * cps, s) !=
+      cudaSuccess)
+    return CP_ECUDA;
+  for (int64_t b0 = 0; b0 < B; b0 += per_launch) {
+    const int64_t nb = (B - b0) < per_launch ? (B - b0) : per_launch;
+    int Ni = (int)N, Ki = (int)K, scene0 = (int)b0;
+    DevParams Pc = P;
+    void* args[] = {(void*)&cost, (void*)&ldc, (void*)&slab, (void*)&nbr, (void*)&v, (void*)&Pc,
+                    (void*)&Ni, (void*)&Ki, (void*)&cps, (void*)&scene0, (void*)&order32,
+                    (void*)&gains, (void*)&objective, (void*)&partials, (void*)&counters,
+                    (void*)&status};
+    cudaError_t e = cudaLaunchCooperativeKernel((const void*)fn, dim3((unsigned)(nb * cps)),
+                                                dim3(SGS_THREADS), args, smem, s);
+    note_launch();
+    if (e != cudaSuccess) return CP_ECUDA;
+  }
+  return CP_OK;
+}
+
+int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
+               const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
+               int32_t* order32, float* gains, double* objective, uint64_t* partials,
+               uint32_t* counters, int* status, cudaStream_t s) {
+  auto* part = reinterpret_cast<unsigned long long*>(partials);
+  if (P.g < N)
+    return sgs_launch_impl<true>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
+                                 part, counters, status, s);
+  return sgs_launch_impl<false>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
+                                part, counters, status, s);
+}
+
+// Upper bound of the partial slots the launcher may use: 2 * B * cps with
+// cps <= ceil(N / SGS_WARPS).
+int64_t sgs_partials_count(int64_t B, int64_t N) {
+  return 2 * B * ((N + SGS_WARPS - 1) / SGS_WARPS);
+}
+
+// ---------------------------------------------------------------------------
+// Barrier self-test: n_blocks co-resident blocks wait for `expected`
+// arrivals; with expected > n_blocks the bounded wait must run out.
+// ---------------------------------------------------------------------------
+__global__ void k_barrier_selftest(uint32_t* ctr, uint32_t expected, int* status,
+                                   uint64_t timeout_ns) {
+  grid_barrier(ctr, expected, status, timeout_ns);
+}
+
+int launch_barrier_selftest(int n_blocks, int expected, uint64_t timeout_ns, uint32_t* ctr,
+                            int* status, cudaStream_t s) {
+  DeviceInfo di;
+  if (device_info(&di) != CP_OK) return CP_ECUDA;
+  if (n_blocks < 1 || n_blocks > di.sm_count || expected < 0) return CP_EINVAL;
+  if (cudaMemsetAsync(ctr, 0, sizeof(uint32_t), s) != cudaSuccess) return CP_ECUDA;
+  if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return CP_ECUDA;
+  uint32_t exp_u = (uint32_t)expected;
+  void* args[] = {(void*)&ctr, (void*)&exp_u, (void*)&status, (void*)&timeout_ns};
+  cudaError_t e = cudaLaunchCooperativeKernel((const void*)k_barrier_selftest, dim3(n_blocks),
+                                              dim3(64), args, 0, s);
+  note_launch();
+  return cuda_status(e);
+}
+
+// ---------------------------------------------------------------------------
+// Ascending sort of K indices per scene (bitonic, shared memory).
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(1024) k_sort_kept(const int32_t* __restrict__ idx32, int K, int L,
+                                                    int64_t* __restrict__ kept,
+                                                    int64_t* __restrict__ order64) {
+  extern __shared__ int32_t sk[];
+  const int b = blockIdx.x;
+  const int32_t* in = idx32 + (size_t)b * K;
+  for (int i = threadIdx.x; i < L; i += blockDim.x) sk[i] = i < K ? in[i] : INT32_MAX;
+  if (order64)
+    for (int i = threadIdx.x; i < K; i += blockDim.x) order64[(size_t)b * K + i] = in[i];
+  __syncthreads();
+  for (int size = 2; size <= L; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < (L >> 1); i += blockDim.x) {
+        const int a = 2 * i - (i & (stride - 1));
+        const int c = a + stride;
+        const bool up = (a & size) == 0;
+        const int32_t x = sk[a], y = sk[c];
+        if ((x > y) == up) { sk[a] = y; sk[c] = x; }
+      }
+      __syncthreads();
+    }
+  }
+  for (int i = threadIdx.x; i < K; i += blockDim.x) kept[(size_t)b * K + i] = sk[i];
+}
+
+int launch_sort_kept(const int32_t* idx32, int64_t B, int64_t K, int64_t* kept, int64_t* order64,
+                     cudaStream_t s) {
+  int L = 2;
+  while (L < K) L <<= 1;
+  const size_t smem = sizeof(int32_t) * (size_t)L;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(k_sort_kept, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+          cudaSuccess)
+    return CP_ECUDA;
+  k_sort_kept<<<(unsigned)B, 1024, smem, s>>>(idx32, (int)K, L, kept, order64);
+  return last_launch_status();
+}
+
+}  // namespace cp
