@@ -292,6 +292,10 @@ typedef enum {
 int coverprune_profile_enable(int on);
 int coverprune_profile_read(double* ms, int64_t* launches, int n);
 
+/* Description of the last CP_ECUDA returned on the calling thread: which
+ * step failed and the CUDA error name ("" if none).  Host only. */
+const char* coverprune_last_error(void);
+
 /* Library version: major * 10000 + minor * 100 + patch. */
 int coverprune_version(void);
 

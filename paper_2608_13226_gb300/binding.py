@@ -25,14 +25,17 @@ EXPORTS = ("cp_default_params", "coverprune_budget", "coverprune_workspace_size"
            "coverprune_status_string", "coverprune_check", "coverprune_cost",
            "coverprune_select", "coverprune_lite_select", "coverprune_knn",
            "coverprune_gather", "coverprune_barrier_selftest", "coverprune_profile_enable",
-           "coverprune_profile_read", "coverprune_version")
+           "coverprune_profile_read", "coverprune_last_error", "coverprune_version")
 STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output")
 
 
 class CoverPruneError(RuntimeError):
     def __init__(self, status: int, what: str):
         self.status = status
-        super().__init__(f"{what}: {status_string(status)} (status {status})")
+        msg = f"{what}: {status_string(status)} (status {status})"
+        if status == CP_ECUDA:
+            msg += f": {_lib().coverprune_last_error().decode()}"
+        super().__init__(msg)
 
 
 class _CpParams(C.Structure):
@@ -110,10 +113,13 @@ def _lib():
         lib.coverprune_knn.argtypes = [P, I64, I64, I64, P, P, P, SZ, P]
         lib.coverprune_gather.argtypes = [P, I32, P, P, I64, I64, I64, P, I64, P, P, P, P, P]
         lib.coverprune_barrier_selftest.argtypes = [C.c_int32, C.c_int32, C.c_float, P, SZ, P]
+        lib.coverprune_last_error.argtypes = []
+        lib.coverprune_last_error.restype = C.c_char_p
         lib.coverprune_profile_enable.argtypes = [I32]
         lib.coverprune_profile_read.argtypes = [P, P, I32]
         for fn in EXPORTS:
-            if fn not in ("cp_default_params", "coverprune_budget", "coverprune_status_string"):
+            if fn not in ("cp_default_params", "coverprune_budget", "coverprune_status_string",
+                          "coverprune_last_error"):
                 getattr(lib, fn).restype = I32
         _L = lib
         return lib

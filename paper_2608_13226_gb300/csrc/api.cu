@@ -2,6 +2,7 @@
 // validation (nothing is launched on bad input), workspace planning and the
 // launch sequence of each entry point.
 #include <math.h>
+#include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
 
@@ -35,6 +36,13 @@ static std::vector<StageEvents> g_prof_events;
 static thread_local int t_stage = CP_STAGE_PREP;
 
 void note_launch() { g_launches[t_stage].fetch_add(1, std::memory_order_relaxed); }
+
+static thread_local char t_last_error[256] = "";
+
+void note_cuda_error(const char* where, cudaError_t e) {
+  snprintf(t_last_error, sizeof(t_last_error), "%s: %s (%s)", where, cudaGetErrorName(e),
+           cudaGetErrorString(e));
+}
 
 // Marks the kernels launched while it lives as belonging to `stage`; with
 // profiling on, brackets them with CUDA events on the call's stream.
@@ -312,6 +320,8 @@ const char* coverprune_status_string(int status) {
 
 int coverprune_version(void) { return 100; }
 
+const char* coverprune_last_error(void) { return t_last_error; }
+
 int coverprune_workspace_size(int op, int64_t B, int64_t N, int64_t D, int64_t K, int dtype,
                               const cp_params* p, size_t* bytes) {
   if (!bytes) return CP_EINVAL;
@@ -335,9 +345,10 @@ int coverprune_workspace_size(int op, int64_t B, int64_t N, int64_t D, int64_t K
 int coverprune_check(const void* ws, cp_stream_t stream) {
   if (!ws) return CP_EINVAL;
   cudaStream_t s = (cudaStream_t)stream;
-  if (cudaStreamSynchronize(s) != cudaSuccess) return CP_ECUDA;
+  CP_TRY(cuda_status(cudaStreamSynchronize(s), "coverprune_check: stream"));
   int st = 0;
-  if (cudaMemcpy(&st, ws, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return CP_ECUDA;
+  CP_TRY(cuda_status(cudaMemcpy(&st, ws, sizeof(int), cudaMemcpyDeviceToHost),
+                     "coverprune_check: status copy"));
   return st;
 }
 

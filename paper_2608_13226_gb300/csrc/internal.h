@@ -129,11 +129,19 @@ constexpr int64_t kMaxKnnN = 49152;
 
 // Counts one kernel launch under the calling thread's current stage.
 void note_launch();
-inline int cuda_status(cudaError_t e) { return e == cudaSuccess ? CP_OK : CP_ECUDA; }
-// After every <<<>>> launch: count it and report launch errors.
-inline int last_launch_status() {
-  note_launch();
-  return cuda_status(cudaGetLastError());
+// Records "where: CUDA error name" as the calling thread's last error.
+void note_cuda_error(const char* where, cudaError_t e);
+inline int cuda_status(cudaError_t e, const char* where = "cuda call") {
+  if (e == cudaSuccess) return CP_OK;
+  note_cuda_error(where, e);
+  (void)cudaGetLastError();  // do not let a failed call resurface at the next launch
+  return CP_ECUDA;
 }
+// After every <<<>>> launch: count it and report launch errors.
+inline int launch_status(const char* where) {
+  note_launch();
+  return cuda_status(cudaGetLastError(), where);
+}
+#define last_launch_status() launch_status(__func__)
 
 }  // namespace cp

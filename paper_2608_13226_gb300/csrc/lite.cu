@@ -64,8 +64,9 @@ int launch_morton(const float* pos, const SceneStats* stats, const DevParams& P,
   while (L < N) L <<= 1;
   const size_t smem = sizeof(unsigned long long) * (size_t)L;
   if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(k_morton, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-          cudaSuccess)
+      cuda_status(cudaFuncSetAttribute(k_morton, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem),
+                  "launch_morton: smem attribute") != CP_OK)
     return CP_ECUDA;
   k_morton<<<(unsigned)B, 1024, smem, s>>>(pos, stats, P.voxel, (int)N, L, perm);
   return last_launch_status();

@@ -221,17 +221,11 @@ int launch_knn(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr, Sce
   while (list_len < kk) list_len <<= 1;
   if (list_len < 2) list_len = 2;
   const size_t smem = sizeof(unsigned long long) * list_len + sizeof(uint32_t) * (size_t)N;
-  static bool attr_set[64] = {false};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (smem > 48 * 1024 && dev < 64 && !attr_set[dev]) {
-    DeviceInfo di;
-    if (device_info(&di) != CP_OK) return CP_ECUDA;
-    if (cudaFuncSetAttribute(k_knn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             di.max_smem_optin) != cudaSuccess)
-      return CP_ECUDA;
-    attr_set[dev] = true;
-  }
+  if (smem > 48 * 1024 &&
+      cuda_status(cudaFuncSetAttribute(k_knn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem),
+                  "launch_knn: smem attribute") != CP_OK)
+    return CP_ECUDA;
   dim3 grid((unsigned)N, (unsigned)B);
   k_knn<<<grid, KNN_THREADS, smem, s>>>(pos, (int)N, kk, list_len, nbr, stats);
   return last_launch_status();

@@ -50,7 +50,7 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
   float* sm_v = sm_m + ncols;                                    // [ncols] capacity v_j
   uint32_t* chosen = reinterpret_cast<uint32_t*>(sm_v + ncols);  // [ceil(N/32)] bitset
   __shared__ unsigned long long s_best[SGS_WARPS];
-  __shared__ int s_pick;
+  __shared__ int s_pick, s_bad;
   __shared__ float s_gain;
 
   const int b = scene0 + blockIdx.x / cps;
@@ -133,19 +133,29 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
       unsigned long long m = 0ull;
       const unsigned long long* pp = part + ((size_t)par * nscenes + (b - scene0)) * cps;
       for (int i = lane; i < cps; i += 32) {
-        const unsigned long long x = __ldcg(pp + i);
+        // each reading lane acquires: a weak load may be served a stale copy
+        const unsigned long long x = ld_acquire_u64(pp + i);
         m = x > m ? x : m;
       }
       m = warp_max_u64(m);
       if (lane == 0) {
-        s_pick = (int)(0xFFFFFFFFu - (uint32_t)(m & 0xFFFFFFFFull));
+        const int pk = (int)(0xFFFFFFFFu - (uint32_t)(m & 0xFFFFFFFFull));
+        s_pick = pk;
         s_gain = __uint_as_float((uint32_t)(m >> 32));
+        // decided once, before anyone updates the state: a winner must be an
+        // unselected token (never expected to fail)
+        s_bad = pk < 0 || pk >= N || (chosen[pk >> 5] & (1u << (pk & 31))) != 0u;
       }
     }
     __syncthreads();
     const int pick = s_pick;
-    if (pick < 0 || pick >= N || (chosen[pick >> 5] & (1u << (pick & 31)))) {
-      if (threadIdx.x == 0) set_status(status, CP_EDEVICE);  // never expected
+    if (s_bad) {
+      if (threadIdx.x == 0 && atomicCAS(status, 0, CP_EDEVICE) == 0) {
+        status[4] = step;  // where it happened, for diagnosis
+        status[5] = b;
+        status[6] = c;
+        status[7] = pick;
+      }
       alive = false;
       break;
     }
@@ -199,10 +209,12 @@ static int sgs_launch_impl(const float* cost, int64_t ldc, const float* slab, co
   const size_t smem = 2 * sizeof(float) * (size_t)ncols + sizeof(uint32_t) * (size_t)((N + 31) / 32);
   auto fn = k_sgs<LOCAL>;
   if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+      cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                  "launch_sgs: smem attribute") != CP_OK)
     return CP_ECUDA;
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SGS_THREADS, smem) != cudaSuccess)
+  if (cuda_status(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, SGS_THREADS, smem),
+                  "launch_sgs: occupancy") != CP_OK)
     return CP_ECUDA;
   if (per_sm < 1) return CP_EUNSUPPORTED;
   const int64_t slots = (int64_t)per_sm * di.sm_count;
@@ -212,9 +224,12 @@ static int sgs_launch_impl(const float* cost, int64_t ldc, const float* slab, co
   const int64_t max_cps = (N + SGS_WARPS - 1) / SGS_WARPS;
   if (cps > max_cps) cps = (int)max_cps;
   if (cps < 1) cps = 1;
-  if (cudaMemsetAsync(counters, 0, sizeof(uint32_t) * (size_t)B, s) != cudaSuccess) return CP_ECUDA;
-  if (cudaMemsetAsync(partials, 0, sizeof(unsigned long long) * 2 * (size_t)per_launch * cps, s) !=
-      cudaSuccess)
+  if (cuda_status(cudaMemsetAsync(counters, 0, sizeof(uint32_t) * (size_t)B, s),
+                  "launch_sgs: counters") != CP_OK)
+    return CP_ECUDA;
+  if (cuda_status(cudaMemsetAsync(partials, 0,
+                                  sizeof(unsigned long long) * 2 * (size_t)per_launch * cps, s),
+                  "launch_sgs: partials") != CP_OK)
     return CP_ECUDA;
   for (int64_t b0 = 0; b0 < B; b0 += per_launch) {
     const int64_t nb = (B - b0) < per_launch ? (B - b0) : per_launch;
@@ -227,7 +242,7 @@ static int sgs_launch_impl(const float* cost, int64_t ldc, const float* slab, co
     cudaError_t e = cudaLaunchCooperativeKernel((const void*)fn, dim3((unsigned)(nb * cps)),
                                                 dim3(SGS_THREADS), args, smem, s);
     note_launch();
-    if (e != cudaSuccess) return CP_ECUDA;
+    if (cuda_status(e, "launch_sgs: cooperative launch") != CP_OK) return CP_ECUDA;
   }
   return CP_OK;
 }
@@ -308,8 +323,9 @@ int launch_sort_kept(const int32_t* idx32, int64_t B, int64_t K, int64_t* kept, 
   while (L < K) L <<= 1;
   const size_t smem = sizeof(int32_t) * (size_t)L;
   if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(k_sort_kept, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-          cudaSuccess)
+      cuda_status(cudaFuncSetAttribute(k_sort_kept, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem),
+                  "launch_sort_kept: smem attribute") != CP_OK)
     return CP_ECUDA;
   k_sort_kept<<<(unsigned)B, 1024, smem, s>>>(idx32, (int)K, L, kept, order64);
   return last_launch_status();

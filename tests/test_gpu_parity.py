@@ -208,6 +208,23 @@ def test_sgs_deterministic_and_batched(orc):
             assert torch.equal(one[k], a[k][i]), (i, k)
 
 
+@pytest.mark.parametrize("g", [0, 9])
+def test_sgs_batch32_launch_shape(g):
+    """32 scenes in one call: the launch shape of the benchmark (several
+    co-resident blocks per SM and per scene).  Every scene must equal its
+    own single-scene call, whose launch shape differs."""
+    scs = [scene("short_clip", sd, N=600, D=64) for sd in range(4)]
+    f, pos, fr = batch_to_dev(scs * 8)
+    K = 150
+    prm = cp.Params(g=g)
+    a = cp.coverprune_select(f, pos, fr, K, prm)
+    assert cp.coverprune_check(a["ws"]) == cp.CP_OK, host(a["ws"][:32].view(torch.int32))
+    singles = [cp.coverprune_select(*to_dev(s), K, prm) for s in scs]
+    for b in range(32):
+        for k in ("kept", "order", "gains", "objective"):
+            assert torch.equal(a[k][b], singles[b % 4][k]), (b, k)
+
+
 def test_sgs_small_edges():
     for N in (1, 2, 3):
         f = torch.randn(N, 8, device="cuda").to(torch.bfloat16)
