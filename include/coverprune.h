@@ -236,6 +236,27 @@ int coverprune_knn(const float* pos, int64_t B, int64_t N, int64_t k, int32_t* n
                    float* diameter, void* ws, size_t ws_bytes, cp_stream_t stream);
 
 /*
+ * coverprune_knn_noalloc -- coverprune_knn for callers that cannot allocate
+ * device memory.  The paper has no counterpart: this is a deployment
+ * variant of the neighbour step above, for hosts that own every device
+ * buffer themselves (a fixed, sealed memory pool; a plugin without access
+ * to an allocator) and can pass inputs and outputs but no workspace.
+ *   Same arguments, results and ordering as coverprune_knn, without ws.
+ *   Its scratch is a fixed array inside the library (65,792 bytes on every
+ *   GPU that loads the library, kept until the process exits): at most
+ *   1024 scenes per call; more returns CP_EUNSUPPORTED (see
+ *   coverprune_last_error).  It calls no allocating routine.
+ *   The first call on each device looks up the array's device address once
+ *   (a runtime query made with that device current); make that first call
+ *   before any stream capture.
+ *   All calls share the array and each call rewrites the part it reads, so
+ *   consecutive calls are independent; calls that overlap on the GPU
+ *   (concurrent streams or host threads on one device) race on it.
+ */
+int coverprune_knn_noalloc(const float* pos, int64_t B, int64_t N, int64_t k, int32_t* nbr,
+                           float* diameter, cp_stream_t stream);
+
+/*
  * coverprune_gather -- compaction of the kept tokens (the pruned visual
  * input of Sec. 3.2).
  *   feats_out [B, K, D] = feats[b, kept[b, k], :] (byte copy, same dtype)

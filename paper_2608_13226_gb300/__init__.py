@@ -9,7 +9,8 @@ generator used by the tests and the benchmark.
 from .binding import (CP_BF16, CP_EINVAL, CP_ETIMEOUT, CP_EUNSUPPORTED, CP_EWORKSPACE, CP_F32,
                       CP_OK, CP_OP_COST, CP_OP_KNN, CP_OP_LITE, CP_OP_SELECT, EXPORTS, CoverPruneError,
                       Params, coverprune_barrier_selftest, coverprune_budget, coverprune_check,
-                      coverprune_cost, coverprune_gather, coverprune_knn, coverprune_lite_select,
+                      coverprune_cost, coverprune_gather, coverprune_knn, coverprune_knn_noalloc,
+                      coverprune_lite_select,
                       coverprune_select, coverprune_version, coverprune_workspace_size,
                       library_path, load, status_string, workspace, coverprune_profile_enable,
                       coverprune_profile_read, STAGES)

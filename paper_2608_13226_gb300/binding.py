@@ -24,6 +24,7 @@ CP_OP_COST, CP_OP_SELECT, CP_OP_LITE, CP_OP_KNN = 0, 1, 2, 3
 EXPORTS = ("cp_default_params", "coverprune_budget", "coverprune_workspace_size",
            "coverprune_status_string", "coverprune_check", "coverprune_cost",
            "coverprune_select", "coverprune_lite_select", "coverprune_knn",
+           "coverprune_knn_noalloc",
            "coverprune_gather", "coverprune_barrier_selftest", "coverprune_profile_enable",
            "coverprune_profile_read", "coverprune_last_error", "coverprune_version")
 STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output")
@@ -111,6 +112,7 @@ def _lib():
         lib.coverprune_lite_select.argtypes = [P, I32, P, P, I64, I64, I64, I64, PP, P, P, P, P,
                                                SZ, P]
         lib.coverprune_knn.argtypes = [P, I64, I64, I64, P, P, P, SZ, P]
+        lib.coverprune_knn_noalloc.argtypes = [P, I64, I64, I64, P, P, P]
         lib.coverprune_gather.argtypes = [P, I32, P, P, I64, I64, I64, P, I64, P, P, P, P, P]
         lib.coverprune_barrier_selftest.argtypes = [C.c_int32, C.c_int32, C.c_float, P, SZ, P]
         lib.coverprune_last_error.argtypes = []
@@ -305,6 +307,24 @@ def coverprune_knn(pos, k: int, *, diameter=True, ws=None):
     if unbatched:
         return nbr[0], (dia[0] if dia is not None else None)
     return nbr, dia
+
+
+def coverprune_knn_noalloc(pos, nbr, diameter=None) -> None:
+    """coverprune_knn into caller-provided outputs, with no workspace: for
+    hosts that cannot allocate device memory (the library uses a fixed
+    internal scratch; at most 1024 scenes per call).  nbr is int32
+    [B, N, k] (or [N, k]), diameter float32 [B] (or a 1-element tensor)."""
+    if pos.dim() == 2:
+        pos = pos.unsqueeze(0)
+        nbr = nbr.unsqueeze(0)
+    if not pos.is_cuda or not pos.is_contiguous() or pos.dtype != torch.float32:
+        raise ValueError("pos must be a contiguous float32 CUDA tensor [B,N,3]")
+    if nbr.dtype != torch.int32 or not nbr.is_contiguous():
+        raise ValueError("nbr must be a contiguous int32 tensor [B,N,k]")
+    B, N, _ = pos.shape
+    k = nbr.shape[-1]
+    _check(_lib().coverprune_knn_noalloc(_ptr(pos), B, N, k, _ptr(nbr), _ptr(diameter),
+                                         _stream()), "coverprune_knn_noalloc")
 
 
 def coverprune_gather(feats, pos, frame, kept, *, status=None, out=None):

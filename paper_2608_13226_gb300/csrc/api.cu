@@ -39,6 +39,8 @@ void note_launch() { g_launches[t_stage].fetch_add(1, std::memory_order_relaxed)
 
 static thread_local char t_last_error[256] = "";
 
+void note_message(const char* msg) { snprintf(t_last_error, sizeof(t_last_error), "%s", msg); }
+
 void note_cuda_error(const char* where, cudaError_t e) {
   snprintf(t_last_error, sizeof(t_last_error), "%s: %s (%s)", where, cudaGetErrorName(e),
            cudaGetErrorString(e));

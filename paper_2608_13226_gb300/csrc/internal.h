@@ -143,5 +143,13 @@ inline int launch_status(const char* where) {
   return cuda_status(cudaGetLastError(), where);
 }
 #define last_launch_status() launch_status(__func__)
+// Records a plain message as the calling thread's last error.
+void note_message(const char* msg);
+
+#define CP_TRY_STATUS(x)          \
+  do {                            \
+    int _st = (x);                \
+    if (_st != CP_OK) return _st; \
+  } while (0)
 
 }  // namespace cp
