@@ -285,7 +285,7 @@ def run_ours(args, rank, world, local_rank, raw):
     sgs_launch_ms = sgs_ms / max(sgs_launches, 1)
     launches_per_step = max(sgs_launches // args.steps, 1)
     sgs_gbs = (sgs_bytes_per_step / launches_per_step) / (sgs_launch_ms / 1000.0) / 1e9
-    traffic = read_traffic("sgs")
+    traffic = read_traffic(B * K // launches_per_step)
     roofline = {"bound": "hbm", "kernel": "k_sgs<dense>", "achieved": round(sgs_gbs, 1),
                 "peak": hbm, "unit": "GB/s", "frac": round(sgs_gbs / hbm, 4),
                 "traffic": traffic, "peak_source": peak_kind,
@@ -420,18 +420,25 @@ def run_ours(args, rank, world, local_rank, raw):
         dist.destroy_process_group()
 
 
-def read_traffic(kernel: str):
-    """DRAM bytes per launch from the committed ncu summary of this kernel,
-    if one exists for the current build (a line 'traffic_bytes_per_launch: X')."""
-    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
+def read_traffic(scene_steps: int):
+    """DRAM bytes of one dense-SGS launch, scaled from the committed ncu
+    record (profiles/sgs_traffic.txt) by scene-steps; None when the kernel
+    source has changed since the counters were taken."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "sgs_traffic.txt")
     try:
+        rec = {}
         for line in open(path):
-            if line.startswith("traffic_bytes_per_launch:"):
-                v = line.split(":", 1)[1].strip()
-                return None if v in ("", "null") else float(v)
-    except OSError:
-        pass
-    return None
+            if ":" in line and not line.startswith("#"):
+                k, v = line.split(":", 1)
+                rec[k.strip()] = v.strip()
+        src = b"".join(open(os.path.join(ROOT, "paper_2608_13226_gb300", "csrc", f), "rb").read()
+                       for f in ("sgs.cu", "common.cuh"))
+        if hashlib.sha256(src).hexdigest()[:16] != rec.get("source_sha256"):
+            return None
+        return float(rec["traffic_bytes_per_scene_step"]) * scene_steps
+    except (OSError, KeyError, ValueError):
+        return None
 
 
 def main():
