@@ -21,6 +21,11 @@ int launch_cost_simt(const void* feats, int dtype, const float* inv, const float
                      const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
                      int64_t N, int64_t D, float* cost, int64_t ldc, cudaStream_t s);
 int64_t sgs_partials_count(int64_t B, int64_t N);
+int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64_t N, int64_t D,
+                          SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s);
+int launch_cost_tc(const void* feats, const float4* tok, const int32_t* frame,
+                   const SceneNorms* norms, const DevParams& P, int64_t B, int64_t N, int64_t D,
+                   float* cost, int64_t ldc, int* status, uint64_t timeout_ns, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Stage timing and launch counting.
@@ -105,18 +110,23 @@ int device_info(DeviceInfo* out) {
   return CP_OK;
 }
 
-int launch_gram_minmax(const void* feats, int dtype, const float* inv, int64_t B, int64_t N,
-                       int64_t D, SceneStats* stats, int* status, uint64_t timeout_ns,
-                       cudaStream_t s) {
-  (void)status;
-  (void)timeout_ns;
+// bf16 features: tcgen05 tensor cores; fp32 features: fp32 FMA tiles (TF32
+// would round the features to 10 mantissa bits).
+int launch_gram_minmax(const void* feats, int dtype, const float* inv, const float4* tok,
+                       int64_t B, int64_t N, int64_t D, SceneStats* stats, int* status,
+                       uint64_t timeout_ns, cudaStream_t s) {
+  if (dtype == CP_BF16)
+    return launch_gram_minmax_tc(feats, tok, B, N, D, stats, status, timeout_ns, s);
   return launch_gram_minmax_simt(feats, dtype, inv, B, N, D, stats, s);
 }
 
-int launch_cost(const void* feats, int dtype, const float* inv, const float* pos,
-                const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
-                int64_t N, int64_t D, float* cost, int64_t ldc, int* status, cudaStream_t s) {
-  (void)status;
+int launch_cost(const void* feats, int dtype, const float* inv, const float4* tok,
+                const float* pos, const int32_t* frame, const SceneNorms* norms,
+                const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
+                int* status, cudaStream_t s) {
+  if (dtype == CP_BF16)
+    return launch_cost_tc(feats, tok, frame, norms, P, B, N, D, cost, ldc, status, P.timeout_ns,
+                          s);
   return launch_cost_simt(feats, dtype, inv, pos, frame, norms, P, B, N, D, cost, ldc, s);
 }
 
@@ -175,7 +185,7 @@ static DevParams dev_params(const cp_params* p, int64_t N) {
 // Workspace plan.  Every region starts on a 256-byte boundary.
 // ---------------------------------------------------------------------------
 struct Plan {
-  size_t hdr, counters, stats, norms, inv, nbr, r, v;
+  size_t hdr, counters, stats, norms, inv, tok, nbr, r, v;
   size_t cost, slab, partials, order32;           // select
   size_t perm, prefix, gs, proto, score;          // lite
   size_t total;
@@ -199,6 +209,7 @@ static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d,
   pl->stats = take(sizeof(SceneStats) * (size_t)B);
   pl->norms = take(sizeof(SceneNorms) * (size_t)B);
   pl->inv = take(sizeof(float) * BN);
+  pl->tok = take(sizeof(float4) * BN);
   pl->nbr = take(sizeof(int32_t) * BN * (size_t)d.kk);
   pl->r = take(sizeof(float) * BN);
   pl->v = take(sizeof(float) * BN);
@@ -252,13 +263,14 @@ static int run_front(const void* feats, int dtype, const float* pos, const int32
     Stage st(CP_STAGE_PREP, s);
     CP_TRY(cuda_status(cudaMemsetAsync(status, 0, sizeof(int), s)));
     CP_TRY(launch_scene_stats(pos, frame, B, N, stats, s));
-    CP_TRY(launch_inv_norms(feats, dtype, B, N, D, at<float>(ws, pl.inv), s));
+    CP_TRY(launch_inv_norms(feats, dtype, pos, B, N, D, at<float>(ws, pl.inv),
+                            at<float4>(ws, pl.tok), s));
     CP_TRY(launch_knn(pos, B, N, d.kk, at<int32_t>(ws, pl.nbr), stats, s));
   }
   {
     Stage st(CP_STAGE_GRAM, s);
-    CP_TRY(launch_gram_minmax(feats, dtype, at<float>(ws, pl.inv), B, N, D, stats, status,
-                              d.timeout_ns, s));
+    CP_TRY(launch_gram_minmax(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), B, N,
+                              D, stats, status, d.timeout_ns, s));
   }
   Stage st(CP_STAGE_PREP, s);
   CP_TRY(launch_finalize_norms(stats, B, at<SceneNorms>(ws, pl.norms), norms_out, s));
@@ -373,8 +385,8 @@ int coverprune_cost(const void* feats, int dtype, const float* pos, const int32_
   const SceneNorms* nm = at<SceneNorms>(ws, pl.norms);
   if (cost) {
     Stage st(CP_STAGE_COST, s);
-    CP_TRY(launch_cost(feats, dtype, at<float>(ws, pl.inv), pos, frame, nm, d, B, N, D, cost, N,
-                       at<int>(ws, pl.hdr), s));
+    CP_TRY(launch_cost(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), pos, frame,
+                       nm, d, B, N, D, cost, N, at<int>(ws, pl.hdr), s));
   }
   if (capacity) {
     Stage st(CP_STAGE_CAPACITY, s);
@@ -415,7 +427,8 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
   float* C = at<float>(ws, pl.cost);
   {
     Stage st(CP_STAGE_COST, s);
-    CP_TRY(launch_cost(feats, dtype, inv, pos, frame, nm, d, B, N, D, C, pl.ldc, status, s));
+    CP_TRY(launch_cost(feats, dtype, inv, at<float4>(ws, pl.tok), pos, frame, nm, d, B, N, D, C,
+                       pl.ldc, status, s));
   }
   int32_t* order32 = at<int32_t>(ws, pl.order32);
   {

@@ -1,4 +1,4 @@
-// K2/K3 for fp32 features: Gram tiles with fp32 FMA (TF32 tensor cores would
+// K2/K3 for fp32 features (bf16 features use gram_tc.cu): Gram tiles with fp32 FMA (TF32 tensor cores would
 // round the features to 10 mantissa bits, far outside the fp32 tolerance),
 // with two epilogues:
 //   MINMAX  max and min of cos(f_i, f_j) over the pairs of the tile (the
@@ -132,13 +132,9 @@ int launch_gram_minmax_simt(const void* feats, int dtype, const float* inv, int6
   const unsigned nt = (unsigned)((N + ST_BM - 1) / ST_BM);
   dim3 grid(nt, nt, (unsigned)B);
   DevParams P{};
-  if (dtype == CP_BF16)
-    k_gram_simt<__nv_bfloat16, EPI_MINMAX><<<grid, ST_THREADS, 0, s>>>(
-        (const __nv_bfloat16*)feats, inv, nullptr, nullptr, nullptr, P, (int)N, (int)D, nullptr, 0,
-        stats);
-  else
-    k_gram_simt<float, EPI_MINMAX><<<grid, ST_THREADS, 0, s>>>(
-        (const float*)feats, inv, nullptr, nullptr, nullptr, P, (int)N, (int)D, nullptr, 0, stats);
+  if (dtype != CP_F32) return CP_EINVAL;  // bf16 features run on the tensor cores
+  k_gram_simt<float, EPI_MINMAX><<<grid, ST_THREADS, 0, s>>>(
+      (const float*)feats, inv, nullptr, nullptr, nullptr, P, (int)N, (int)D, nullptr, 0, stats);
   return last_launch_status();
 }
 
@@ -147,12 +143,9 @@ int launch_cost_simt(const void* feats, int dtype, const float* inv, const float
                      int64_t N, int64_t D, float* cost, int64_t ldc, cudaStream_t s) {
   const unsigned nt = (unsigned)((N + ST_BM - 1) / ST_BM);
   dim3 grid(nt, nt, (unsigned)B);
-  if (dtype == CP_BF16)
-    k_gram_simt<__nv_bfloat16, EPI_COST><<<grid, ST_THREADS, 0, s>>>(
-        (const __nv_bfloat16*)feats, inv, pos, frame, norms, P, (int)N, (int)D, cost, ldc, nullptr);
-  else
-    k_gram_simt<float, EPI_COST><<<grid, ST_THREADS, 0, s>>>(
-        (const float*)feats, inv, pos, frame, norms, P, (int)N, (int)D, cost, ldc, nullptr);
+  if (dtype != CP_F32) return CP_EINVAL;  // bf16 features run on the tensor cores
+  k_gram_simt<float, EPI_COST><<<grid, ST_THREADS, 0, s>>>(
+      (const float*)feats, inv, pos, frame, norms, P, (int)N, (int)D, cost, ldc, nullptr);
   return last_launch_status();
 }
 

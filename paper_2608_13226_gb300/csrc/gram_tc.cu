@@ -1,0 +1,544 @@
+// K2/K3 for bf16 features on the 5th-generation tensor cores (tcgen05 + TMEM).
+//
+// The feature Gram G = F F^T of one scene is the method's only dense
+// contraction (the cosine of Eq. fst_metrics).  Two epilogues consume it:
+//   MINMAX  max and min of cos(f_i, f_j) over the pairs i <= j (the feature
+//           normaliser of Sec. 3.3) -- only the tiles on or above the
+//           diagonal run, no output but two atomics per warp
+//   COST    the FST cost of Eq. fst_cost, written row-major with stride ldc
+//
+// One persistent CTA per SM, 6 warps:
+//   warp 0      TMA producer: 128x64 (A) and 256x64 (B) bf16 boxes, 128-byte
+//               swizzle, into a 4-stage shared-memory ring (48 KB a stage)
+//   warp 1      allocates 512 TMEM columns; lane 0 issues
+//               tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) into
+//               one of two 128x256 fp32 accumulators (double buffer)
+//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 32 columns at a time, FST
+//               arithmetic in registers, 16-byte stores (or the min/max)
+// Stage hand-offs use mbarriers; the accumulator hand-off uses
+// tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
+// time limit: on expiry the kernel records CP_ETIMEOUT, stops issuing work,
+// waits (bounded) for the copies and MMAs it already issued, frees its TMEM
+// and returns.
+#include <cuda.h>
+
+#include "common.cuh"
+
+namespace cp {
+namespace {
+
+constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 4;
+constexpr int TC_THREADS = 192;
+constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
+constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;  // 32 KB
+constexpr uint32_t TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
+constexpr uint32_t TC_TMEM_COLS = 512;              // 2 accumulators x 256 fp32 columns
+constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES + 1024;  // + alignment slack
+
+enum { TC_MINMAX = 0, TC_COST = 1 };
+
+// Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16,
+// both K-major, M = 128, N = 256.
+constexpr uint32_t kIdesc = (1u << 4)              // D format: f32
+                            | (1u << 7)            // A format: bf16
+                            | (1u << 10)           // B format: bf16
+                            | ((uint32_t)(TC_BN >> 3) << 17)   // N >> 3
+                            | ((uint32_t)(TC_BM >> 4) << 24);  // M >> 4
+
+struct TcArgs {
+  const float4* tok;      // [B*N] (x, y, z, 1/||f||)
+  const int32_t* frame;   // [B*N]
+  const SceneNorms* norms;
+  DevParams P;
+  float* cost;
+  int64_t ldc;
+  SceneStats* stats;
+  int* status;
+  int N, B, TI, TJ, num_kb, tiles_per_scene, total_tiles;
+  uint64_t timeout_ns;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+// ---- mbarrier ---------------------------------------------------------------
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+// Waits for the phase of parity `parity` to complete.  Gives up when the
+// block has aborted or this wait exceeds timeout_ns (then aborts the block).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          uint64_t timeout_ns, int* status) {
+  if (mbar_test(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  uint32_t spins = 0;
+  while (!mbar_test(bar, parity)) {
+    if ((++spins & 15u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > timeout_ns) {
+        set_status(status, CP_ETIMEOUT);
+        *abort_flag = 1;
+        return false;
+      }
+    }
+  }
+  return true;
+}
+
+// ---- TMA ---------------------------------------------------------------------
+__device__ __forceinline__ void tma_load_3d(const CUtensorMap* map, uint64_t* bar, uint32_t dst,
+                                            int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// ---- tcgen05 -------------------------------------------------------------------
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row
+// groups 1024 bytes apart (the layout a 128-byte-wide TMA box with
+// SWIZZLE_128B writes).  Leading-byte offset unused for this layout.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4)       // start address >> 4
+         | ((uint64_t)1 << 16)                     // leading byte offset (unused) = 16 B
+         | ((uint64_t)(1024 >> 4) << 32)           // stride byte offset = 1024 B
+         | ((uint64_t)1 << 46)                     // descriptor version (fixed 0b001)
+         | ((uint64_t)2 << 61);                    // swizzle mode: 128 B
+}
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Warp-reduce a scene's running max / min cosine and merge it into stats.
+__device__ __forceinline__ void flush_minmax(SceneStats* st, float cmax, float cmin) {
+  for (int o = 16; o > 0; o >>= 1) {
+    cmax = fmaxf(cmax, __shfl_xor_sync(0xFFFFFFFFu, cmax, o));
+    cmin = fminf(cmin, __shfl_xor_sync(0xFFFFFFFFu, cmin, o));
+  }
+  if ((threadIdx.x & 31) == 0 && cmax >= cmin) {
+    atomicMax(&st->cos_max_key, f2key(cmax));
+    atomicMin(&st->cos_min_key, f2key(cmin));
+  }
+}
+
+// Tile t of the schedule -> (scene b, row tile I, column tile J).  MINMAX
+// visits only J >= I/2 (tiles holding a pair i <= j); COST visits all.
+template <int MODE>
+__device__ __forceinline__ void tile_coords(const TcArgs& a, int t, int& b, int& I, int& J) {
+  b = t / a.tiles_per_scene;
+  int r = t - b * a.tiles_per_scene;
+  if (MODE == TC_COST) {
+    I = r / a.TJ;
+    J = r - I * a.TJ;
+  } else {
+    I = 0;
+    while (r >= a.TJ - (I >> 1)) {
+      r -= a.TJ - (I >> 1);
+      ++I;
+    }
+    J = (I >> 1) + r;
+  }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    k_gram_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+              const TcArgs a) {
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES];
+  __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2];
+  __shared__ uint32_t s_tmem_base;
+  __shared__ volatile int s_abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t smem_base = (smem_u32(smem_raw) + 1023u) & ~1023u;  // 1024-B aligned ring
+
+  if (threadIdx.x == 0) {
+    s_abort = 0;
+    for (int s = 0; s < TC_STAGES; ++s) {
+      mbar_init(&full_bar[s], 1);   // producer's arrive + the TMA bytes
+      mbar_init(&empty_bar[s], 1);  // one tcgen05.commit
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull_bar[i], 1);     // one tcgen05.commit
+      mbar_init(&tempty_bar[i], 128);  // every epilogue thread
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    tma_prefetch_desc(&mapA);
+    tma_prefetch_desc(&mapB);
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&s_tmem_base)),
+                 "r"(TC_TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = s_tmem_base;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t pending = 0;        // stages holding a load not yet seen consumed
+      uint32_t pend_parity = 0;    // parity of that load's full phase, per stage bit
+      for (int t = blockIdx.x; t < a.total_tiles && !s_abort; t += gridDim.x) {
+        int b, I, J;
+        tile_coords<MODE>(a, t, b, I, J);
+        for (int kb = 0; kb < a.num_kb; ++kb) {
+          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
+          pending &= ~(1u << stage);
+          const uint32_t sa = smem_base + (uint32_t)stage * TC_STAGE_BYTES;
+          mbar_arrive_expect_tx(&full_bar[stage], TC_STAGE_BYTES);
+          tma_load_3d(&mapA, &full_bar[stage], sa, kb * TC_BK, I * TC_BM, b);
+          tma_load_3d(&mapB, &full_bar[stage], sa + TC_A_BYTES, kb * TC_BK, J * TC_BN, b);
+          pending |= 1u << stage;
+          pend_parity = (pend_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == TC_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (s_abort) {
+        // let the copies already issued land before the block exits
+        const uint64_t drain = globaltimer_ns() + 50000000ull;
+        for (int s = 0; s < TC_STAGES; ++s)
+          if (pending & (1u << s))
+            while (!mbar_test(&full_bar[s], (pend_parity >> s) & 1u) && globaltimer_ns() < drain) {
+            }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      uint64_t* last_commit = nullptr;
+      uint32_t last_parity = 0;
+      for (int t = blockIdx.x; t < a.total_tiles && !s_abort; t += gridDim.x) {
+        if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
+        tc_fence_after();
+        const uint32_t tmem_d = tmem_base + (uint32_t)(acc * TC_BN);
+        bool ok = true;
+        for (int kb = 0; kb < a.num_kb; ++kb) {
+          if (!mbar_wait(&full_bar[stage], phase, &s_abort, a.timeout_ns, a.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_base + (uint32_t)stage * TC_STAGE_BYTES;
+          const uint64_t adesc = sw128_desc(sa), bdesc = sw128_desc(sa + TC_A_BYTES);
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)  // 32 bytes further along K per step
+            umma_bf16(tmem_d, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k),
+                      (kb > 0 || k > 0) ? 1u : 0u);
+          umma_commit(&empty_bar[stage]);  // frees the stage when these MMAs finish
+          last_commit = &empty_bar[stage];
+          last_parity = phase;
+          if (++stage == TC_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(&tfull_bar[acc]);  // accumulator ready for the epilogue
+        last_commit = &tfull_bar[acc];
+        last_parity = acc_phase;
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+      if (s_abort && last_commit) {
+        // the MMAs already issued must finish before TMEM is freed
+        const uint64_t drain = globaltimer_ns() + 50000000ull;
+        while (!mbar_test(last_commit, last_parity) && globaltimer_ns() < drain) {
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;          // TMEM lanes 32q .. 32q+31 belong to this warp
+    const int r = q * 32 + lane;     // row of the tile
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    float cmax = -INFINITY, cmin = INFINITY;
+    int cur_b = -1;
+    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
+      // lane 0 waits, the warp follows it (keeps the warp converged for the
+      // .sync.aligned TMEM loads below)
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull_bar[acc], acc_phase, &s_abort, a.timeout_ns, a.status);
+      ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      int b, I, J;
+      tile_coords<MODE>(a, t, b, I, J);
+      if (MODE == TC_MINMAX && b != cur_b) {
+        if (cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
+        cur_b = b;
+        cmax = -INFINITY;
+        cmin = INFINITY;
+      }
+      const int gi = I * TC_BM + r;
+      const bool row_ok = gi < a.N;
+      const size_t sb = (size_t)b * a.N;
+      float4 ti = make_float4(0.f, 0.f, 0.f, 0.f);
+      int taui = 0;
+      if (row_ok) {
+        ti = __ldg(a.tok + sb + gi);
+        taui = __ldg(a.frame + sb + gi);
+      }
+      SceneNorms nm;
+      float* crow = nullptr;
+      if (MODE == TC_COST) {
+        nm = a.norms[b];
+        crow = a.cost + (sb + (size_t)(row_ok ? gi : 0)) * (size_t)a.ldc;
+      }
+      const uint32_t row_taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN);
+#pragma unroll 1
+      for (int c = 0; c < TC_BN / 32; ++c) {
+        uint32_t v[32];
+        __syncwarp();
+        tmem_ld32(row_taddr + (uint32_t)(c * 32), v);
+        const int j0 = J * TC_BN + c * 32;
+        if (row_ok) {
+          if (MODE == TC_MINMAX) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const int j = j0 + e;
+              if (j < a.N) {
+                const float inv_j = __ldg(&a.tok[sb + j].w);
+                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * inv_j);
+                if (j == gi && ti.w > 0.0f) cv = 1.0f;  // cos(f, f) = 1 exactly
+                cmax = fmaxf(cmax, cv);
+                cmin = fminf(cmin, cv);
+              }
+            }
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const int j = j0 + e;
+              float out = 0.0f;  // pad columns N <= j < ldc hold 0
+              if (j < a.N) {
+                const float4 tj = __ldg(a.tok + sb + j);
+                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * tj.w);
+                if (j == gi && ti.w > 0.0f) cv = 1.0f;
+                const float d2 = sqdist_rn(ti.x, ti.y, ti.z, tj.x, tj.y, tj.z);
+                out = fst_cost_from(cv, d2, taui, __ldg(a.frame + sb + j), nm, a.P);
+              }
+              v[e] = __float_as_uint(out);
+            }
+            if ((a.ldc & 3) == 0 && j0 + 32 <= a.ldc) {
+              float4* dst = reinterpret_cast<float4*>(crow + j0);
+#pragma unroll
+              for (int e = 0; e < 8; ++e)
+                dst[e] = make_float4(__uint_as_float(v[4 * e]), __uint_as_float(v[4 * e + 1]),
+                                     __uint_as_float(v[4 * e + 2]), __uint_as_float(v[4 * e + 3]));
+            } else {
+#pragma unroll
+              for (int e = 0; e < 32; ++e)
+                if (j0 + e < a.ldc) crow[j0 + e] = __uint_as_float(v[e]);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tempty_bar[acc]);  // accumulator free for the MMA warp
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+    if (MODE == TC_MINMAX && cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TC_TMEM_COLS)
+                 : "memory");
+  }
+}
+
+}  // namespace
+}  // namespace cp
+
+#include <limits.h>
+
+#include <mutex>
+
+namespace cp {
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+    else
+      (void)cudaGetLastError();
+  });
+  return fn;
+}
+
+// 3D view [B][N][D] of the bf16 features; box = 64 features x box_rows tokens
+// x 1 scene, 128-byte swizzle; rows past N (and features past D) read as 0.
+int make_feature_map(CUtensorMap* map, const void* feats, int64_t B, int64_t N, int64_t D,
+                     uint32_t box_rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) {
+    note_message("launch_gram_tc: cuTensorMapEncodeTiled unavailable");
+    return CP_ECUDA;
+  }
+  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)N, (cuuint64_t)B};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)N * (cuuint64_t)D * 2};
+  const cuuint32_t box[3] = {(cuuint32_t)TC_BK, box_rows, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(feats), dims,
+                         strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    note_message("launch_gram_tc: cuTensorMapEncodeTiled rejected the feature layout");
+    return CP_ECUDA;
+  }
+  return CP_OK;
+}
+
+template <int MODE>
+int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const SceneNorms* norms,
+              const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
+              SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s) {
+  DeviceInfo di;
+  if (device_info(&di) != CP_OK) return CP_ECUDA;
+  alignas(64) CUtensorMap mapA, mapB;
+  CP_TRY_STATUS(make_feature_map(&mapA, feats, B, N, D, TC_BM));
+  CP_TRY_STATUS(make_feature_map(&mapB, feats, B, N, D, TC_BN));
+  TcArgs a{};
+  a.tok = tok;
+  a.frame = frame;
+  a.norms = norms;
+  a.P = P;
+  a.cost = cost;
+  a.ldc = ldc;
+  a.stats = stats;
+  a.status = status;
+  a.N = (int)N;
+  a.B = (int)B;
+  a.TI = (int)((N + TC_BM - 1) / TC_BM);
+  a.TJ = (int)((N + TC_BN - 1) / TC_BN);
+  a.num_kb = (int)((D + TC_BK - 1) / TC_BK);
+  int64_t tps = 0;
+  if (MODE == TC_COST) {
+    tps = (int64_t)a.TI * a.TJ;
+  } else {
+    for (int I = 0; I < a.TI; ++I) tps += a.TJ - (I >> 1);
+  }
+  const int64_t total = tps * B;
+  if (total > INT_MAX) return CP_EUNSUPPORTED;
+  a.tiles_per_scene = (int)tps;
+  a.total_tiles = (int)total;
+  a.timeout_ns = timeout_ns;
+  const int grid = (int)(total < di.sm_count ? total : di.sm_count);
+  auto fn = k_gram_tc<MODE>;
+  if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)TC_SMEM),
+                  "launch_gram_tc: smem attribute") != CP_OK)
+    return CP_ECUDA;
+  fn<<<grid, TC_THREADS, TC_SMEM, s>>>(mapA, mapB, a);
+  return last_launch_status();
+}
+
+}  // namespace
+
+int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64_t N, int64_t D,
+                          SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s) {
+  DevParams P{};
+  return launch_tc<TC_MINMAX>(feats, tok, nullptr, nullptr, P, B, N, D, nullptr, 0, stats, status,
+                              timeout_ns, s);
+}
+
+int launch_cost_tc(const void* feats, const float4* tok, const int32_t* frame,
+                   const SceneNorms* norms, const DevParams& P, int64_t B, int64_t N, int64_t D,
+                   float* cost, int64_t ldc, int* status, uint64_t timeout_ns, cudaStream_t s) {
+  return launch_tc<TC_COST>(feats, tok, frame, norms, P, B, N, D, cost, ldc, nullptr, status,
+                            timeout_ns, s);
+}
+
+}  // namespace cp

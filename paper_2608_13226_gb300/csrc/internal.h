@@ -62,18 +62,19 @@ int device_info(DeviceInfo* out);
 // atomically reduced fields of `stats`.
 int launch_scene_stats(const float* pos, const int32_t* frame, int64_t B, int64_t N,
                        SceneStats* stats, cudaStream_t s);
-// K0: inverse feature norms inv[b*N + j] (0 for a zero feature).
-int launch_inv_norms(const void* feats, int dtype, int64_t B, int64_t N, int64_t D,
-                     float* inv, cudaStream_t s);
+// K0: inverse feature norms inv[b*N + j] (0 for a zero feature) and the
+// packed per-token record tok[b*N + j] = (x, y, z, inv) the Gram epilogues read.
+int launch_inv_norms(const void* feats, int dtype, const float* pos, int64_t B, int64_t N,
+                     int64_t D, float* inv, float4* tok, cudaStream_t s);
 // K1: per token the kk nearest other tokens by (fp32 d^2, index) into
 // nbr[(b*N + j)*kk + q]; also the scene's largest squared distance.
 int launch_knn(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
                cudaStream_t s);
 // K2 (fp32 SIMT and bf16 tensor-core variants): max and min cosine over all
 // pairs into stats.
-int launch_gram_minmax(const void* feats, int dtype, const float* inv, int64_t B, int64_t N,
-                       int64_t D, SceneStats* stats, int* status, uint64_t timeout_ns,
-                       cudaStream_t s);
+int launch_gram_minmax(const void* feats, int dtype, const float* inv, const float4* tok,
+                       int64_t B, int64_t N, int64_t D, SceneStats* stats, int* status,
+                       uint64_t timeout_ns, cudaStream_t s);
 // Scene diameter sqrt(max d^2) from stats into out[b].
 int launch_diameter(const SceneStats* stats, int64_t B, float* out, cudaStream_t s);
 // Normalisers from stats.  Optionally also the public [B, 6] float copy.
@@ -81,9 +82,10 @@ int launch_finalize_norms(const SceneStats* stats, int64_t B, SceneNorms* norms,
                           float* norms_out, cudaStream_t s);
 // K3: the FST cost C[b][s][t] into cost + b*N*ldc + s*ldc + t for t < N;
 // columns N <= t < ldc are written as 0.
-int launch_cost(const void* feats, int dtype, const float* inv, const float* pos,
-                const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
-                int64_t N, int64_t D, float* cost, int64_t ldc, int* status, cudaStream_t s);
+int launch_cost(const void* feats, int dtype, const float* inv, const float4* tok,
+                const float* pos, const int32_t* frame, const SceneNorms* norms,
+                const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
+                int* status, cudaStream_t s);
 // K4: capacity score r and capacity v (Eqs. fst_capacity_score, fst_capacity).
 int launch_capacity(const void* feats, int dtype, const float* inv, const float* pos,
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,

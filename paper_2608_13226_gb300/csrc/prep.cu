@@ -67,8 +67,10 @@ int launch_scene_stats(const float* pos, const int32_t* frame, int64_t B, int64_
 // K0b: inv[j] = 1 / ||f_j|| (0 for a zero feature), one warp per token.
 // ---------------------------------------------------------------------------
 template <typename T>
-__global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ F, int64_t rows, int D,
-                                                   float* __restrict__ inv) {
+__global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ F,
+                                                   const float* __restrict__ pos, int64_t rows,
+                                                   int D, float* __restrict__ inv,
+                                                   float4* __restrict__ tok) {
   const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -82,17 +84,22 @@ __global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ F, int6
     for (int i = 0; i < V; ++i) acc = fmaf(x[i], x[i], acc);
   }
   acc = warp_sum(acc);
-  if (lane == 0) inv[row] = acc > 0.0f ? 1.0f / sqrtf(acc) : 0.0f;
+  if (lane == 0) {
+    const float iv = acc > 0.0f ? 1.0f / sqrtf(acc) : 0.0f;
+    inv[row] = iv;
+    if (tok) tok[row] = make_float4(pos[3 * row], pos[3 * row + 1], pos[3 * row + 2], iv);
+  }
 }
 
-int launch_inv_norms(const void* feats, int dtype, int64_t B, int64_t N, int64_t D, float* inv,
-                     cudaStream_t s) {
+int launch_inv_norms(const void* feats, int dtype, const float* pos, int64_t B, int64_t N,
+                     int64_t D, float* inv, float4* tok, cudaStream_t s) {
   const int64_t rows = B * N;
   const unsigned grid = (unsigned)((rows + 7) / 8);
   if (dtype == CP_BF16)
-    k_inv_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)feats, rows, (int)D, inv);
+    k_inv_norms<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)feats, pos, rows,
+                                                     (int)D, inv, tok);
   else
-    k_inv_norms<float><<<grid, 256, 0, s>>>((const float*)feats, rows, (int)D, inv);
+    k_inv_norms<float><<<grid, 256, 0, s>>>((const float*)feats, pos, rows, (int)D, inv, tok);
   return last_launch_status();
 }
 
