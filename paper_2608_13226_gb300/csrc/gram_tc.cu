@@ -7,14 +7,17 @@
 //           diagonal run, no output but two atomics per warp
 //   COST    the FST cost of Eq. fst_cost, written row-major with stride ldc
 //
-// One persistent CTA per SM, 6 warps:
+// One persistent CTA per SM, 10 warps:
 //   warp 0      TMA producer: 128x64 (A) and 256x64 (B) bf16 boxes, 128-byte
 //               swizzle, into a 4-stage shared-memory ring (48 KB a stage)
 //   warp 1      allocates 512 TMEM columns; lane 0 issues
 //               tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) into
 //               one of two 128x256 fp32 accumulators (double buffer)
-//   warps 2..5  epilogue: tcgen05.ld 32 lanes x 32 columns at a time, FST
-//               arithmetic in registers, 16-byte stores (or the min/max)
+//   warps 2..9  epilogue: warps w and w+4 share TMEM lane quadrant w%4 and
+//               split the 256 columns; tcgen05.ld 32 lanes x 32 columns at a
+//               time, FST arithmetic in registers, 16-byte stores (or the
+//               min/max); the 32 columns' token data is staged per warp in
+//               shared memory
 // Stage hand-offs use mbarriers; the accumulator hand-off uses
 // tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
 // time limit: on expiry the kernel records CP_ETIMEOUT, stops issuing work,
@@ -28,7 +31,8 @@ namespace cp {
 namespace {
 
 constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 4;
-constexpr int TC_THREADS = 192;
+constexpr int TC_EPI_WARPS = 8;                     // two per TMEM lane quadrant
+constexpr int TC_THREADS = 64 + 32 * TC_EPI_WARPS;  // producer, MMA, epilogue
 constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
 constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;  // 32 KB
 constexpr uint32_t TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
@@ -165,6 +169,20 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// FST cost of one pair (Eq. fst_cost) for the tensor-core path: as
+// fst_cost_from, with the distance from rsqrtf and log(1 + x) from __log2f
+// (both within ~1e-7 absolute here, far inside the bf16 parity bar).
+__device__ __forceinline__ float fst_cost_fast(float cosv, float d2, int tau_s, int tau_t,
+                                               const SceneNorms& nm, const DevParams& P,
+                                               float log2_scale) {
+  const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
+  const float dx = d2 > 0.0f ? d2 * rsqrtf(d2) : 0.0f;
+  const float tx = __log2f(1.0f + P.kappa * (dx * nm.x_rinv)) * log2_scale;
+  const int dt = tau_s - tau_t;
+  const float tt = dt > 0 ? (float)dt * nm.t_rinv : 0.0f;
+  return P.lambda_f * tf + P.lambda_x * tx + P.lambda_tau * tt;
+}
+
 // Warp-reduce a scene's running max / min cosine and merge it into stats.
 __device__ __forceinline__ void flush_minmax(SceneStats* st, float cmax, float cmin) {
   for (int o = 16; o > 0; o >>= 1) {
@@ -205,6 +223,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2];
   __shared__ uint32_t s_tmem_base;
   __shared__ volatile int s_abort;
+  __shared__ float4 s_col[TC_EPI_WARPS][32];  // per epilogue warp: (x, y, z, 1/||f||)
+  __shared__ int s_tau[TC_EPI_WARPS][32];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t smem_base = (smem_u32(smem_raw) + 1023u) & ~1023u;  // 1024-B aligned ring
@@ -217,7 +237,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);     // one tcgen05.commit
-      mbar_init(&tempty_bar[i], 128);  // every epilogue thread
+      mbar_init(&tempty_bar[i], 32 * TC_EPI_WARPS);  // every epilogue thread
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
@@ -321,8 +341,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;          // TMEM lanes 32q .. 32q+31 belong to this warp
-    const int r = q * 32 + lane;     // row of the tile
+    const int q = warp & 3;                        // TMEM lane quadrant of this warp
+    const int half = (warp - 2) / 4;               // which 128 of the 256 columns
+    const int ew = warp - 2;                       // epilogue warp index (staging slot)
+    const int r = q * 32 + lane;                   // row of the tile
+    const float log2_scale = 0.69314718055994531f * a.P.inv_log1p_kappa;
     int acc = 0;
     uint32_t acc_phase = 0;
     float cmax = -INFINITY, cmin = INFINITY;
@@ -350,7 +373,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       int taui = 0;
       if (row_ok) {
         ti = __ldg(a.tok + sb + gi);
-        taui = __ldg(a.frame + sb + gi);
+        if (MODE == TC_COST) taui = __ldg(a.frame + sb + gi);
       }
       SceneNorms nm;
       float* crow = nullptr;
@@ -360,19 +383,31 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       }
       const uint32_t row_taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN);
 #pragma unroll 1
-      for (int c = 0; c < TC_BN / 32; ++c) {
-        uint32_t v[32];
-        __syncwarp();
-        tmem_ld32(row_taddr + (uint32_t)(c * 32), v);
+      for (int c = half * 4; c < half * 4 + 4; ++c) {
         const int j0 = J * TC_BN + c * 32;
+        // stage the 32 columns' token data (one column per lane, coalesced)
+        {
+          const int jl = j0 + lane;
+          float4 tj = make_float4(0.f, 0.f, 0.f, 0.f);
+          int tauj = 0;
+          if (jl < a.N) {
+            tj = __ldg(a.tok + sb + jl);
+            if (MODE == TC_COST) tauj = __ldg(a.frame + sb + jl);
+          }
+          __syncwarp();
+          s_col[ew][lane] = tj;
+          s_tau[ew][lane] = tauj;
+          __syncwarp();
+        }
+        uint32_t v[32];
+        tmem_ld32(row_taddr + (uint32_t)(c * 32), v);
         if (row_ok) {
           if (MODE == TC_MINMAX) {
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
               const int j = j0 + e;
               if (j < a.N) {
-                const float inv_j = __ldg(&a.tok[sb + j].w);
-                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * inv_j);
+                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * s_col[ew][e].w);
                 if (j == gi && ti.w > 0.0f) cv = 1.0f;  // cos(f, f) = 1 exactly
                 cmax = fmaxf(cmax, cv);
                 cmin = fminf(cmin, cv);
@@ -384,11 +419,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               const int j = j0 + e;
               float out = 0.0f;  // pad columns N <= j < ldc hold 0
               if (j < a.N) {
-                const float4 tj = __ldg(a.tok + sb + j);
+                const float4 tj = s_col[ew][e];
                 float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * tj.w);
                 if (j == gi && ti.w > 0.0f) cv = 1.0f;
-                const float d2 = sqdist_rn(ti.x, ti.y, ti.z, tj.x, tj.y, tj.z);
-                out = fst_cost_from(cv, d2, taui, __ldg(a.frame + sb + j), nm, a.P);
+                const float dx = ti.x - tj.x, dy = ti.y - tj.y, dz = ti.z - tj.z;
+                const float d2 = dx * dx + dy * dy + dz * dz;
+                out = fst_cost_fast(cv, d2, taui, s_tau[ew][e], nm, a.P, log2_scale);
               }
               v[e] = __float_as_uint(out);
             }

@@ -222,8 +222,75 @@ __global__ void __launch_bounds__(KNN_THREADS) k_knn(const float* __restrict__ p
   for (int q = threadIdx.x; q < kk; q += KNN_THREADS) out[q] = (int32_t)(list[q] & 0xFFFFFFFFu);
 }
 
+// K1 for kk <= 32: one warp per token.  Each lane scans every 32nd candidate
+// and keeps its KK smallest (d^2 bits, index) keys in registers, sorted; the
+// warp then merges the 32 lists by repeated warp-wide minimum.  The keys are
+// the same total order as the block kernel's, so the lists are identical.
+template <int KK>
+__global__ void __launch_bounds__(256) k_knn_warp(const float* __restrict__ pos, int N, int kk,
+                                                  int32_t* __restrict__ nbr, SceneStats* stats) {
+  const int j = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int b = blockIdx.y;
+  const int lane = threadIdx.x & 31;
+  const float* X = pos + (size_t)b * N * 3;
+  uint32_t dmax = 0u;
+  if (j < N) {
+    const float xj = X[3 * j], yj = X[3 * j + 1], zj = X[3 * j + 2];
+    unsigned long long best[KK];
+#pragma unroll
+    for (int i = 0; i < KK; ++i) best[i] = ~0ull;
+    for (int k = lane; k < N; k += 32) {
+      const float d2 = sqdist_rn(xj, yj, zj, __ldg(X + 3 * k), __ldg(X + 3 * k + 1),
+                                 __ldg(X + 3 * k + 2));
+      const uint32_t bits = __float_as_uint(d2);
+      dmax = max(dmax, bits);
+      const unsigned long long key = ((unsigned long long)bits << 32) | (uint32_t)k;
+      if (k != j && key < best[KK - 1]) {
+        best[KK - 1] = key;
+#pragma unroll
+        for (int i = KK - 1; i > 0; --i) {
+          if (best[i] < best[i - 1]) {
+            const unsigned long long t = best[i];
+            best[i] = best[i - 1];
+            best[i - 1] = t;
+          }
+        }
+      }
+    }
+    int32_t* out = nbr + ((size_t)b * N + j) * kk;
+    for (int q = 0; q < kk; ++q) {
+      const unsigned long long m = warp_min_u64(best[0]);
+      if (lane == 0) out[q] = (int32_t)(m & 0xFFFFFFFFull);
+      if (best[0] == m) {  // keys are unique: exactly one lane pops its head
+#pragma unroll
+        for (int i = 0; i < KK - 1; ++i) best[i] = best[i + 1];
+        best[KK - 1] = ~0ull;
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) dmax = max(dmax, __shfl_xor_sync(0xFFFFFFFFu, dmax, o));
+  __shared__ uint32_t s_dmax[8];
+  if (lane == 0) s_dmax[threadIdx.x >> 5] = dmax;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t m = s_dmax[0];
+    for (int i = 1; i < 8; ++i) m = max(m, s_dmax[i]);
+    atomicMax(&stats[b].d2_max_bits, m);
+  }
+}
+
 int launch_knn(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
                cudaStream_t s) {
+  if (kk <= 32) {
+    dim3 grid((unsigned)((N + 7) / 8), (unsigned)B);
+    if (kk <= 8)
+      k_knn_warp<8><<<grid, 256, 0, s>>>(pos, (int)N, kk, nbr, stats);
+    else if (kk <= 16)
+      k_knn_warp<16><<<grid, 256, 0, s>>>(pos, (int)N, kk, nbr, stats);
+    else
+      k_knn_warp<32><<<grid, 256, 0, s>>>(pos, (int)N, kk, nbr, stats);
+    return last_launch_status();
+  }
   int list_len = 1;
   while (list_len < kk) list_len <<= 1;
   if (list_len < 2) list_len = 2;
