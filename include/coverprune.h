@@ -103,6 +103,12 @@ typedef enum {
  *   timeout_ms                      limit of every device-side wait, after
  *                                   which the kernel records CP_ETIMEOUT and
  *                                   returns (> 0; default 2000)
+ *   sgs_mode                        how SGS finds each step's winner, with
+ *                                   identical results: 0 = lazy (a gain
+ *                                   computed at an earlier step bounds the
+ *                                   current one, so only candidates whose
+ *                                   bound could still win are re-evaluated;
+ *                                   default), 1 = every gain every step
  */
 typedef struct {
   uint32_t struct_size; /* = sizeof(cp_params); set by cp_default_params */
@@ -115,6 +121,7 @@ typedef struct {
   float voxel_m;
   float m0;
   float timeout_ms;
+  int32_t sgs_mode;
 } cp_params;
 
 /* Fills *p with the defaults listed above.  Host only; p must not be NULL. */

@@ -45,7 +45,8 @@ class _CpParams(C.Structure):
                 ("kappa", C.c_float),
                 ("alpha_f", C.c_float), ("alpha_x", C.c_float), ("alpha_tau", C.c_float),
                 ("n_cap", C.c_int32), ("g", C.c_int32), ("capacity_mode", C.c_int32),
-                ("voxel_m", C.c_float), ("m0", C.c_float), ("timeout_ms", C.c_float)]
+                ("voxel_m", C.c_float), ("m0", C.c_float), ("timeout_ms", C.c_float),
+                ("sgs_mode", C.c_int32)]
 
 
 @dataclass
@@ -65,6 +66,7 @@ class Params:
     voxel_m: float = 0.2
     m0: float = 0.0
     timeout_ms: float = 2000.0
+    sgs_mode: int = 0
 
     def _c(self) -> _CpParams:
         p = _CpParams()

@@ -148,6 +148,7 @@ static int check_params(const cp_params* p) {
   if (!(isfinite(p->timeout_ms) && p->timeout_ms > 0.0f)) return CP_EINVAL;
   if (p->n_cap < 0 || p->g < 0) return CP_EINVAL;
   if (p->capacity_mode != 0 && p->capacity_mode != 1) return CP_EINVAL;
+  if (p->sgs_mode != 0 && p->sgs_mode != 1) return CP_EINVAL;
   return CP_OK;
 }
 
@@ -177,6 +178,7 @@ static DevParams dev_params(const cp_params* p, int64_t N) {
   d.g = (p->g == 0 || p->g >= N) ? (int)N : p->g;
   d.kk = d.g < N ? (d.n_cap > d.g - 1 ? d.n_cap : d.g - 1) : d.n_cap;
   d.cap_mode = p->capacity_mode;
+  d.sgs_mode = p->sgs_mode;
   d.timeout_ns = (uint64_t)((double)p->timeout_ms * 1.0e6);
   return d;
 }
@@ -309,6 +311,7 @@ void cp_default_params(cp_params* p) {
   p->voxel_m = 0.2f;
   p->m0 = 0.0f;
   p->timeout_ms = 2000.0f;
+  p->sgs_mode = 0;
 }
 
 int64_t coverprune_budget(double R, int64_t N) {

@@ -6,7 +6,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/coverprune.h"
+#include "coverprune.h"
 
 namespace cp {
 
@@ -20,6 +20,7 @@ struct DevParams {
   int g;       // SGS neighbourhood incl. the token itself; == N means all
   int kk;      // neighbours stored per token = max(n_cap, g-1) (g < N) or n_cap
   int cap_mode;
+  int sgs_mode;  // 0 = lazy evaluation of gains, 1 = every gain every step
   uint64_t timeout_ns;
 };
 

@@ -37,6 +37,81 @@ __device__ __forceinline__ unsigned long long gain_key(float gain, int t) {
   return ((unsigned long long)__float_as_uint(gain) << 32) | (0xFFFFFFFFu - (uint32_t)t);
 }
 
+// One term of gain(t) = sum_j v_j max(m_j - C(t, j), 0), each operation
+// rounded once: the computed gain can only decrease when m decreases, which
+// makes a gain computed at an earlier step an upper bound of the current one.
+__device__ __forceinline__ float gain_term(float acc, float v, float m, float c) {
+  return __fmaf_rn(v, fmaxf(__fsub_rn(m, c), 0.0f), acc);
+}
+
+// gain(t) over a dense padded row (ncols % 4 == 0, pad v = 0).  Lane l sums
+// the float4 chunks l, l+32, l+64, ... in ascending order, then a butterfly:
+// the same fixed order in every kernel that evaluates a gain.  The result is
+// identical in all lanes.
+__device__ __forceinline__ float dense_row_gain(const float* __restrict__ crow,
+                                                const float* sm_m, const float* sm_v, int ncols,
+                                                int lane) {
+  const float4* row = reinterpret_cast<const float4*>(crow);
+  const float4* m4 = reinterpret_cast<const float4*>(sm_m);
+  const float4* v4 = reinterpret_cast<const float4*>(sm_v);
+  const int nq = ncols >> 2;
+  float acc = 0.0f;
+  int q = lane;
+  for (; q + 224 < nq; q += 256) {
+    float4 cs[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) cs[u] = ld_stream_f4(row + q + 32 * u);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const float4 mm = m4[q + 32 * u], vv = v4[q + 32 * u];
+      acc = gain_term(acc, vv.x, mm.x, cs[u].x);
+      acc = gain_term(acc, vv.y, mm.y, cs[u].y);
+      acc = gain_term(acc, vv.z, mm.z, cs[u].z);
+      acc = gain_term(acc, vv.w, mm.w, cs[u].w);
+    }
+  }
+  for (; q < nq; q += 32) {
+    const float4 c0 = ld_stream_f4(row + q);
+    const float4 mm = m4[q], vv = v4[q];
+    acc = gain_term(acc, vv.x, mm.x, c0.x);
+    acc = gain_term(acc, vv.y, mm.y, c0.y);
+    acc = gain_term(acc, vv.z, mm.z, c0.z);
+    acc = gain_term(acc, vv.w, mm.w, c0.w);
+  }
+  return warp_sum(acc);
+}
+
+// gain(t) over the local neighbourhood M_g(t): slab row of g costs, member
+// k = 0 is t itself, members k >= 1 are t's nearest others.
+__device__ __forceinline__ float local_row_gain(const float* __restrict__ srow,
+                                                const int32_t* __restrict__ nb, int t, int g,
+                                                const float* sm_m, const float* sm_v, int lane) {
+  float acc = 0.0f;
+  for (int k = lane; k < g; k += 32) {
+    const int j = k == 0 ? t : nb[k - 1];
+    acc = gain_term(acc, sm_v[j], sm_m[j], srow[k]);
+  }
+  return warp_sum(acc);
+}
+
+// F(S) = sum_j v_j m_j in fp64, in one fixed order whatever the block size
+// (>= 512 threads): thread r < 512 sums j = r, r+512, ...; then 16 warp
+// butterflies; then the 16 warp sums in order.  Every thread of the block
+// must call it; the result is valid in thread 0.
+__device__ __forceinline__ double objective_sum(const float* sm_m, const float* sm_v, int N) {
+  __shared__ double s_part[16];
+  double part = 0.0;
+  if (threadIdx.x < 512)
+    for (int j = threadIdx.x; j < N; j += 512) part += (double)sm_v[j] * (double)sm_m[j];
+  if (threadIdx.x < 512) part = warp_sum(part);
+  if (threadIdx.x < 512 && (threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = part;
+  __syncthreads();
+  double t = 0.0;
+  if (threadIdx.x == 0)
+    for (int i = 0; i < 16; ++i) t += s_part[i];
+  return t;
+}
+
 template <bool LOCAL>
 __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
     const float* __restrict__ cost, int64_t ldc, const float* __restrict__ slab,
@@ -77,43 +152,10 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
     unsigned long long best = 0ull;
     for (int t = gw; t < N; t += nw) {
       if (chosen[t >> 5] & (1u << (t & 31))) continue;
-      float acc = 0.0f;
-      if (!LOCAL) {
-        const float4* row = reinterpret_cast<const float4*>(Cb + (size_t)t * ldc);
-        const float4* m4 = reinterpret_cast<const float4*>(sm_m);
-        const float4* v4 = reinterpret_cast<const float4*>(sm_v);
-        const int nq = ncols >> 2;
-        int q = lane;
-        for (; q + 96 < nq; q += 128) {
-          float4 c0 = ld_stream_f4(row + q), c1 = ld_stream_f4(row + q + 32);
-          float4 c2 = ld_stream_f4(row + q + 64), c3 = ld_stream_f4(row + q + 96);
-          const float4 cs[4] = {c0, c1, c2, c3};
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float4 mm = m4[q + 32 * u], vv = v4[q + 32 * u];
-            acc += vv.x * fmaxf(mm.x - cs[u].x, 0.0f);
-            acc += vv.y * fmaxf(mm.y - cs[u].y, 0.0f);
-            acc += vv.z * fmaxf(mm.z - cs[u].z, 0.0f);
-            acc += vv.w * fmaxf(mm.w - cs[u].w, 0.0f);
-          }
-        }
-        for (; q < nq; q += 32) {
-          const float4 c0 = ld_stream_f4(row + q);
-          const float4 mm = m4[q], vv = v4[q];
-          acc += vv.x * fmaxf(mm.x - c0.x, 0.0f);
-          acc += vv.y * fmaxf(mm.y - c0.y, 0.0f);
-          acc += vv.z * fmaxf(mm.z - c0.z, 0.0f);
-          acc += vv.w * fmaxf(mm.w - c0.w, 0.0f);
-        }
-      } else {
-        const float* srow = Sb + (size_t)t * P.g;
-        const int32_t* nb = NB + (size_t)t * P.kk;
-        for (int k = lane; k < P.g; k += 32) {
-          const int j = k == 0 ? t : nb[k - 1];
-          acc += sm_v[j] * fmaxf(sm_m[j] - srow[k], 0.0f);
-        }
-      }
-      acc = warp_sum(acc);  // identical in every lane
+      const float acc =
+          LOCAL ? local_row_gain(Sb + (size_t)t * P.g, NB + (size_t)t * P.kk, t, P.g, sm_m, sm_v,
+                                 lane)
+                : dense_row_gain(Cb + (size_t)t * ldc, sm_m, sm_v, ncols, lane);
       const unsigned long long key = gain_key(acc, t);
       best = key > best ? key : best;
     }
@@ -182,18 +224,8 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
   }
 
   if (c == 0 && alive && objective) {
-    double part_sum = 0.0;
-    for (int j = threadIdx.x; j < N; j += SGS_THREADS)
-      part_sum += (double)sm_v[j] * (double)sm_m[j];
-    part_sum = warp_sum(part_sum);
-    __shared__ double s_obj[SGS_WARPS];
-    if (lane == 0) s_obj[w] = part_sum;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      double t = 0.0;
-      for (int i = 0; i < SGS_WARPS; ++i) t += s_obj[i];
-      objective[b] = t;
-    }
+    const double F = objective_sum(sm_m, sm_v, N);
+    if (threadIdx.x == 0) objective[b] = F;
   }
 }
 
@@ -247,11 +279,179 @@ static int sgs_launch_impl(const float* cost, int64_t ldc, const float* slab, co
   return CP_OK;
 }
 
+
+// ---------------------------------------------------------------------------
+// Lazy evaluation of the same greedy (exact, bit-identical picks).
+//
+// A gain computed at an earlier step is an upper bound of the current one
+// (gain_term is monotone in m and m only decreases), so the step's winner --
+// the largest (gain, -index) key -- is found without evaluating every
+// candidate: keep the last computed gain ub[t] of every token; a candidate
+// whose bound is exact this step ("fresh") and larger than every other bound
+// is the winner.  One block of 32 warps per scene; warp w owns the
+// candidates [w*S, (w+1)*S).  Each round every warp reports the largest
+// bound of its slice; if the overall largest is fresh the step is decided,
+// otherwise each warp whose slice-best is stale and could still beat the
+// best fresh key recomputes that row.  Step 0 evaluates every candidate.
+// No inter-block synchronisation: blocks are independent scenes.
+// ---------------------------------------------------------------------------
+constexpr int LZ_THREADS = 1024;
+constexpr int LZ_WARPS = LZ_THREADS / 32;
+
+template <bool LOCAL>
+__global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
+    const float* __restrict__ cost, int64_t ldc, const float* __restrict__ slab,
+    const int32_t* __restrict__ nbr, const float* __restrict__ v_all, DevParams P, int N, int K,
+    int32_t* __restrict__ order32, float* __restrict__ gains, double* __restrict__ objective,
+    int* status) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int ncols = LOCAL ? N : (int)ldc;
+  const int nwords = (N + 31) >> 5;
+  float* sm_m = reinterpret_cast<float*>(smem);                 // [ncols] coverage cost
+  float* sm_v = sm_m + ncols;                                   // [ncols] capacity
+  float* ub = sm_v + ncols;                                     // [N] last computed gain
+  uint32_t* chosen = reinterpret_cast<uint32_t*>(ub + N);       // [nwords]
+  uint32_t* fresh = chosen + nwords;                            // [nwords]
+  __shared__ unsigned long long s_wkey[LZ_WARPS];
+  __shared__ int s_wfresh[LZ_WARPS];
+
+  const int b = blockIdx.x;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* v = v_all + (size_t)b * N;
+  const float* Cb = LOCAL ? nullptr : cost + (size_t)b * N * ldc;
+  const float* Sb = LOCAL ? slab + (size_t)b * N * P.g : nullptr;
+  const int32_t* NB = nbr + (size_t)b * N * P.kk;
+
+  for (int j = threadIdx.x; j < ncols; j += LZ_THREADS) {
+    sm_m[j] = j < N ? P.m0 : 0.0f;
+    sm_v[j] = j < N ? v[j] : 0.0f;
+  }
+  for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) chosen[i] = 0u;
+  __syncthreads();
+
+  auto gain_of = [&](int t) -> float {
+    return LOCAL ? local_row_gain(Sb + (size_t)t * P.g, NB + (size_t)t * P.kk, t, P.g, sm_m, sm_v,
+                                  lane)
+                 : dense_row_gain(Cb + (size_t)t * ldc, sm_m, sm_v, ncols, lane);
+  };
+  // step 0: every gain exactly
+  for (int t = w; t < N; t += LZ_WARPS) {
+    const float g0 = gain_of(t);
+    if (lane == 0) ub[t] = g0;
+  }
+  const int S = (N + LZ_WARPS - 1) / LZ_WARPS;
+  const int t_lo = w * S, t_hi = min(N, t_lo + S);
+
+  for (int step = 0; step < K; ++step) {
+    for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) fresh[i] = step == 0 ? ~0u : 0u;
+    __syncthreads();
+    int pick = -1;
+    for (int round = 0; round <= N; ++round) {
+      unsigned long long best = 0ull;
+      for (int t = t_lo + lane; t < t_hi; t += 32)
+        if (!(chosen[t >> 5] & (1u << (t & 31)))) {
+          const unsigned long long key = gain_key(ub[t], t);
+          best = key > best ? key : best;
+        }
+      best = warp_max_u64(best);
+      if (lane == 0) {
+        const int bt = (int)(0xFFFFFFFFu - (uint32_t)(best & 0xFFFFFFFFull));
+        s_wkey[w] = best;
+        s_wfresh[w] = best != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
+      }
+      __syncthreads();
+      unsigned long long G = 0ull, BF = 0ull;
+      for (int i = 0; i < LZ_WARPS; ++i) {
+        const unsigned long long k = s_wkey[i];
+        G = k > G ? k : G;
+        if (s_wfresh[i]) BF = k > BF ? k : BF;
+      }
+      const unsigned long long mine = s_wkey[w];
+      const bool mine_fresh = s_wfresh[w] != 0;
+      __syncthreads();  // s_wkey / s_wfresh are rewritten next round
+      if (G != 0ull && G == BF) {  // the largest bound is exact: the winner
+        pick = (int)(0xFFFFFFFFu - (uint32_t)(G & 0xFFFFFFFFull));
+        break;
+      }
+      if (G == 0ull) break;  // no candidate left (never for K <= N)
+      if (!mine_fresh && mine > BF) {  // this slice's best might still win
+        const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
+        const float g = gain_of(t);
+        if (lane == 0) {
+          ub[t] = g;
+          atomicOr(&fresh[t >> 5], 1u << (t & 31));
+        }
+      }
+      __syncthreads();
+    }
+    // every thread checks the winner before anyone updates the state
+    const bool bad = pick < 0 || pick >= N || (chosen[pick >> 5] & (1u << (pick & 31))) != 0u;
+    __syncthreads();
+    if (bad) {  // never expected; block-uniform (every thread has the same pick)
+      if (threadIdx.x == 0 && atomicCAS(status, 0, CP_EDEVICE) == 0) {
+        status[4] = step;
+        status[5] = b;
+        status[6] = 0;
+        status[7] = pick;
+      }
+      return;
+    }
+    if (threadIdx.x == 0) {
+      chosen[pick >> 5] |= 1u << (pick & 31);
+      order32[(size_t)b * K + step] = pick;
+      if (gains) gains[(size_t)b * K + step] = ub[pick];
+    }
+    // S <- S u {t*} (Eq. sgs_update)
+    if (!LOCAL) {
+      const float* row = Cb + (size_t)pick * ldc;
+      for (int j = threadIdx.x; j < N; j += LZ_THREADS) sm_m[j] = fminf(sm_m[j], __ldg(row + j));
+    } else {
+      const float* srow = Sb + (size_t)pick * P.g;
+      const int32_t* nb = NB + (size_t)pick * P.kk;
+      for (int k = threadIdx.x; k < P.g; k += LZ_THREADS) {
+        const int j = k == 0 ? pick : nb[k - 1];
+        sm_m[j] = fminf(sm_m[j], srow[k]);
+      }
+    }
+    __syncthreads();
+  }
+
+  if (objective) {
+    const double F = objective_sum(sm_m, sm_v, N);
+    if (threadIdx.x == 0) objective[b] = F;
+  }
+}
+
+template <bool LOCAL>
+static int sgs_lazy_launch(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
+                           const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
+                           int32_t* order32, float* gains, double* objective, int* status,
+                           cudaStream_t s) {
+  const int64_t ncols = LOCAL ? N : ldc;
+  const size_t smem = sizeof(float) * (size_t)(2 * ncols + N) +
+                      2 * sizeof(uint32_t) * (size_t)((N + 31) / 32);
+  auto fn = k_sgs_lazy<LOCAL>;
+  if (smem > 48 * 1024 &&
+      cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                  "launch_sgs_lazy: smem attribute") != CP_OK)
+    return CP_ECUDA;
+  fn<<<(unsigned)B, LZ_THREADS, smem, s>>>(cost, ldc, slab, nbr, v, P, (int)N, (int)K, order32,
+                                          gains, objective, status);
+  return last_launch_status();
+}
+
 int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
                int32_t* order32, float* gains, double* objective, uint64_t* partials,
                uint32_t* counters, int* status, cudaStream_t s) {
   auto* part = reinterpret_cast<unsigned long long*>(partials);
+  if (P.sgs_mode == 0) {
+    if (P.g < N)
+      return sgs_lazy_launch<true>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
+                                   status, s);
+    return sgs_lazy_launch<false>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
+                                  status, s);
+  }
   if (P.g < N)
     return sgs_launch_impl<true>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
                                  part, counters, status, s);

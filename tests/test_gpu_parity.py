@@ -225,6 +225,24 @@ def test_sgs_batch32_launch_shape(g):
             assert torch.equal(a[k][b], singles[b % 4][k]), (b, k)
 
 
+@pytest.mark.parametrize("name,N,D,K,g,B", [("tiny", 1024, 256, 102, 0, 1),
+                                             ("short_clip", 1500, 512, 300, 0, 3),
+                                             ("long_video", 2000, 512, 400, 20, 2),
+                                             ("short_clip", 777, 128, 777, 0, 1),
+                                             ("long_video", 3000, 256, 450, 0, 32)])
+def test_sgs_lazy_equals_full_sweep(name, N, D, K, g, B):
+    """Lazy evaluation only skips candidates whose earlier (upper-bound) gain
+    cannot win, so it must reproduce the full sweep bit for bit."""
+    scs = [scene(name, sd, N=N, D=D) for sd in range(min(B, 4))]
+    f, pos, fr = batch_to_dev((scs * B)[:B])
+    lazy = cp.coverprune_select(f, pos, fr, K, cp.Params(g=g, sgs_mode=0))
+    full = cp.coverprune_select(f, pos, fr, K, cp.Params(g=g, sgs_mode=1))
+    assert cp.coverprune_check(lazy["ws"]) == cp.CP_OK
+    assert cp.coverprune_check(full["ws"]) == cp.CP_OK
+    for k in ("kept", "order", "gains", "objective"):
+        assert torch.equal(lazy[k], full[k]), k
+
+
 def test_sgs_small_edges():
     for N in (1, 2, 3):
         f = torch.randn(N, 8, device="cuda").to(torch.bfloat16)
