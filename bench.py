@@ -278,19 +278,26 @@ def run_ours(args, rank, world, local_rank, raw):
     ms_step = max_over_ranks(ev0.elapsed_time(ev1) / args.steps)
     value = B * world / (ms_step / 1000.0)
 
-    # roofline of the dominant kernel (dense SGS sweep) from its own events
+    # roofline of the SGS kernel from its own events and its counted reads:
+    # every gain evaluation reads one padded cost row, every step one row
+    # to update the coverage cost
     hbm, tf_burst, tf_sust, peak_kind = measured_peaks()
+    cstats = cp.coverprune_call_stats(ws)
     sgs_ms, sgs_launches = prof["sgs"]
-    sgs_bytes_per_step = B * K * (N * N * 4 + N * 4)  # C read once per greedy step + row update
-    sgs_launch_ms = sgs_ms / max(sgs_launches, 1)
     launches_per_step = max(sgs_launches // args.steps, 1)
+    ldc = (N + 3) // 4 * 4
+    sgs_bytes_per_step = cstats["gain_evaluations"] * ldc * 4 + B * K * N * 4
+    sgs_launch_ms = sgs_ms / max(sgs_launches, 1)
     sgs_gbs = (sgs_bytes_per_step / launches_per_step) / (sgs_launch_ms / 1000.0) / 1e9
-    traffic = read_traffic(B * K // launches_per_step)
-    roofline = {"bound": "hbm", "kernel": "k_sgs<dense>", "achieved": round(sgs_gbs, 1),
-                "peak": hbm, "unit": "GB/s", "frac": round(sgs_gbs / hbm, 4),
-                "traffic": traffic, "peak_source": peak_kind,
-                "algorithmic_bytes_per_launch": sgs_bytes_per_step // launches_per_step,
-                "avg_launch_ms": round(sgs_launch_ms, 3)}
+    roofline_sgs = {"bound": "hbm", "kernel": "k_sgs_lazy<dense>", "achieved": round(sgs_gbs, 1),
+                    "peak": hbm, "unit": "GB/s", "frac": round(sgs_gbs / hbm, 4),
+                    "traffic": read_traffic("k_sgs_lazy", cstats["gain_evaluations"]),
+                    "peak_source": peak_kind,
+                    "algorithmic_bytes_per_launch": sgs_bytes_per_step // launches_per_step,
+                    "avg_launch_ms": round(sgs_launch_ms, 3),
+                    "gain_evaluations_per_step": cstats["gain_evaluations"],
+                    "rounds_per_step": cstats["rounds"],
+                    "full_sweep_evaluations_per_step": B * (K * N - K * (K - 1) // 2)}
     def tflops(stage, flops_per_call):
         ms, launches = prof[stage]
         if ms <= 0 or launches <= 0:
@@ -301,13 +308,45 @@ def run_ours(args, rank, world, local_rank, raw):
     cost_tf = tflops("cost", B * 2.0 * N * N * D)            # full N x N x D product
     gram_tf = tflops("gram", B * 1.0 * N * (N + 1) * D)      # the pairs i <= j once
     roofline_gemm = {"bound": "tensor", "unit": "TFLOP/s", "peak": tf_burst,
-                     "cost_gemm": {"achieved": cost_tf and round(cost_tf, 1),
+                     "cost_gemm": {"kernel": "k_gram_tc<COST>",
+                                   "achieved": cost_tf and round(cost_tf, 1),
                                    "frac": cost_tf and round(cost_tf / tf_burst, 4),
-                                   "flops_per_launch": B * 2 * N * N * D},
-                     "normaliser_gemm": {"achieved": gram_tf and round(gram_tf, 1),
+                                   "flops_per_launch": B * 2 * N * N * D,
+                                   "avg_launch_ms": round(prof["cost"][0] / max(prof["cost"][1], 1), 3)},
+                     "normaliser_gemm": {"kernel": "k_gram_tc<MINMAX>",
+                                         "achieved": gram_tf and round(gram_tf, 1),
                                          "frac": gram_tf and round(gram_tf / tf_burst, 4),
                                          "flops_per_launch": B * N * (N + 1) * D},
                      "peak_source": peak_kind}
+    # the line's roofline is the kernel with the largest share of the step
+    if prof["sgs"][0] >= prof["cost"][0]:
+        roofline = roofline_sgs
+    else:
+        roofline = {"bound": "tensor", "kernel": "k_gram_tc<COST>", "achieved": round(cost_tf, 1),
+                    "peak": tf_burst, "unit": "TFLOP/s", "frac": round(cost_tf / tf_burst, 4),
+                    "traffic": None, "peak_source": peak_kind,
+                    "algorithmic_flops_per_launch": B * 2 * N * N * D}
+
+    # the full sweep (every gain every step), same picks: its HBM roofline
+    prm_full = cp.Params(sgs_mode=1)
+    cp.coverprune_select(feats, pos, fr, K, prm_full, order=False, gains=False, ws=ws, out=out)
+    barrier()
+    cp.coverprune_profile_read()
+    cp.coverprune_profile_enable(True)
+    full_steps = 2
+    for _ in range(full_steps):
+        cp.coverprune_select(feats, pos, fr, K, prm_full, order=False, gains=False, ws=ws, out=out)
+    barrier()
+    cp.coverprune_profile_enable(False)
+    fprof = cp.coverprune_profile_read()
+    fstats = cp.coverprune_call_stats(ws)
+    f_ms = fprof["sgs"][0] / max(fprof["sgs"][1], 1)
+    f_bytes = fstats["gain_evaluations"] * ldc * 4 + B * K * N * 4
+    f_gbs = f_bytes / (f_ms / 1000.0) / 1e9
+    sweep = {"bound": "hbm", "kernel": "k_sgs<dense>", "achieved": round(f_gbs, 1), "peak": hbm,
+             "unit": "GB/s", "frac": round(f_gbs / hbm, 4),
+             "traffic": read_traffic("k_sgs", fstats["gain_evaluations"]),
+             "algorithmic_bytes_per_launch": f_bytes, "avg_launch_ms": round(f_ms, 3)}
     stages = {k: round(v[0] / args.steps, 3) for k, v in prof.items() if v[0] > 0}
     gpu_launches = sum(v[1] for v in prof.values())
 
@@ -411,7 +450,8 @@ def run_ours(args, rank, world, local_rank, raw):
                        "generator": "paper_2608_13226_gb300.scenes long_video, seeds "
                                     f"{rank * B}..{rank * B + B - 1} per rank"},
             "latency_ms": round(latency_ms, 3),
-            "lite": lite, "roofline": roofline, "roofline_gemm": roofline_gemm,
+            "lite": lite, "roofline": roofline, "roofline_sgs": roofline_sgs,
+            "roofline_gemm": roofline_gemm, "sgs_full_sweep": sweep,
             "stages_ms": stages, "gpu_launches": gpu_launches, "e2e": e2e,
             "clocks": clocks, "cpu_baseline": cpu}
     print(json.dumps(line), flush=True)
@@ -420,12 +460,14 @@ def run_ours(args, rank, world, local_rank, raw):
         dist.destroy_process_group()
 
 
-def read_traffic(scene_steps: int):
-    """DRAM bytes of one dense-SGS launch, scaled from the committed ncu
-    record (profiles/sgs_traffic.txt) by scene-steps; None when the kernel
-    source has changed since the counters were taken."""
+def read_traffic(kernel: str, evaluations: int):
+    """DRAM bytes of one SGS launch, scaled from the committed ncu record of
+    that kernel (profiles/<kernel>_traffic.txt: bytes per gain evaluation,
+    which reads one cost row) by the launch's evaluations; None when no
+    record exists or the kernel source has changed since the counters were
+    taken."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", "sgs_traffic.txt")
+    path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
     try:
         rec = {}
         for line in open(path):
@@ -436,7 +478,7 @@ def read_traffic(scene_steps: int):
                        for f in ("sgs.cu", "common.cuh"))
         if hashlib.sha256(src).hexdigest()[:16] != rec.get("source_sha256"):
             return None
-        return float(rec["traffic_bytes_per_scene_step"]) * scene_steps
+        return float(rec["traffic_bytes_per_evaluation"]) * evaluations
     except (OSError, KeyError, ValueError):
         return None
 

@@ -320,6 +320,22 @@ typedef enum {
 int coverprune_profile_enable(int on);
 int coverprune_profile_read(double* ms, int64_t* launches, int n);
 
+/*
+ * Counters of the last coverprune_select that used workspace `ws`
+ * (synchronises `stream` first):
+ *   gain_evaluations  candidate gains computed, over all scenes and steps;
+ *                     each reads one row of the cost (N floats) or of the
+ *                     local slab (g floats)
+ *   rounds            decision rounds over all scenes and steps (lazy mode:
+ *                     a step needs one or more; full sweep: one per step)
+ * Returns CP_OK, CP_EINVAL or CP_ECUDA.
+ */
+typedef struct {
+  uint64_t gain_evaluations;
+  uint64_t rounds;
+} cp_call_stats;
+int coverprune_call_stats(const void* ws, cp_stream_t stream, cp_call_stats* out);
+
 /* Description of the last CP_ECUDA returned on the calling thread: which
  * step failed and the CUDA error name ("" if none).  Host only. */
 const char* coverprune_last_error(void);

@@ -8,7 +8,7 @@ generator used by the tests and the benchmark.
 """
 from .binding import (CP_BF16, CP_EINVAL, CP_ETIMEOUT, CP_EUNSUPPORTED, CP_EWORKSPACE, CP_F32,
                       CP_OK, CP_OP_COST, CP_OP_KNN, CP_OP_LITE, CP_OP_SELECT, EXPORTS, CoverPruneError,
-                      Params, coverprune_barrier_selftest, coverprune_budget, coverprune_check,
+                      Params, coverprune_barrier_selftest, coverprune_budget, coverprune_call_stats, coverprune_check,
                       coverprune_cost, coverprune_gather, coverprune_knn, coverprune_knn_noalloc,
                       coverprune_lite_select,
                       coverprune_select, coverprune_version, coverprune_workspace_size,

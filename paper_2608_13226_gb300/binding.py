@@ -26,7 +26,8 @@ EXPORTS = ("cp_default_params", "coverprune_budget", "coverprune_workspace_size"
            "coverprune_select", "coverprune_lite_select", "coverprune_knn",
            "coverprune_knn_noalloc",
            "coverprune_gather", "coverprune_barrier_selftest", "coverprune_profile_enable",
-           "coverprune_profile_read", "coverprune_last_error", "coverprune_version")
+           "coverprune_profile_read", "coverprune_last_error", "coverprune_call_stats",
+           "coverprune_version")
 STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output")
 
 
@@ -47,6 +48,10 @@ class _CpParams(C.Structure):
                 ("n_cap", C.c_int32), ("g", C.c_int32), ("capacity_mode", C.c_int32),
                 ("voxel_m", C.c_float), ("m0", C.c_float), ("timeout_ms", C.c_float),
                 ("sgs_mode", C.c_int32)]
+
+
+class _CallStats(C.Structure):
+    _fields_ = [("gain_evaluations", C.c_uint64), ("rounds", C.c_uint64)]
 
 
 @dataclass
@@ -117,6 +122,7 @@ def _lib():
         lib.coverprune_knn_noalloc.argtypes = [P, I64, I64, I64, P, P, P]
         lib.coverprune_gather.argtypes = [P, I32, P, P, I64, I64, I64, P, I64, P, P, P, P, P]
         lib.coverprune_barrier_selftest.argtypes = [C.c_int32, C.c_int32, C.c_float, P, SZ, P]
+        lib.coverprune_call_stats.argtypes = [P, P, C.POINTER(_CallStats)]
         lib.coverprune_last_error.argtypes = []
         lib.coverprune_last_error.restype = C.c_char_p
         lib.coverprune_profile_enable.argtypes = [I32]
@@ -371,6 +377,14 @@ def coverprune_profile_read() -> dict:
     la = (C.c_int64 * n)()
     _check(_lib().coverprune_profile_read(ms, la, n), "coverprune_profile_read")
     return {name: (float(ms[i]), int(la[i])) for i, name in enumerate(STAGES)}
+
+
+def coverprune_call_stats(ws) -> dict:
+    """{"gain_evaluations", "rounds"} of the last coverprune_select on ws."""
+    out = _CallStats()
+    _check(_lib().coverprune_call_stats(_ptr(ws), _stream(), C.byref(out)),
+           "coverprune_call_stats")
+    return {"gain_evaluations": int(out.gain_evaluations), "rounds": int(out.rounds)}
 
 
 def coverprune_version() -> int:

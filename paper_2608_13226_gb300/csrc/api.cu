@@ -263,7 +263,7 @@ static int run_front(const void* feats, int dtype, const float* pos, const int32
   SceneStats* stats = at<SceneStats>(ws, pl.stats);
   {
     Stage st(CP_STAGE_PREP, s);
-    CP_TRY(cuda_status(cudaMemsetAsync(status, 0, sizeof(int), s)));
+    CP_TRY(cuda_status(cudaMemsetAsync(status, 0, kStatusBytes, s), "status block"));
     CP_TRY(launch_scene_stats(pos, frame, B, N, stats, s));
     CP_TRY(launch_inv_norms(feats, dtype, pos, B, N, D, at<float>(ws, pl.inv),
                             at<float4>(ws, pl.tok), s));
@@ -367,6 +367,18 @@ int coverprune_check(const void* ws, cp_stream_t stream) {
   CP_TRY(cuda_status(cudaMemcpy(&st, ws, sizeof(int), cudaMemcpyDeviceToHost),
                      "coverprune_check: status copy"));
   return st;
+}
+
+int coverprune_call_stats(const void* ws, cp_stream_t stream, cp_call_stats* out) {
+  if (!ws || !out) return CP_EINVAL;
+  CP_TRY(cuda_status(cudaStreamSynchronize((cudaStream_t)stream), "coverprune_call_stats: stream"));
+  unsigned long long v[2] = {0, 0};
+  CP_TRY(cuda_status(cudaMemcpy(v, static_cast<const unsigned char*>(ws) + kCallStatsOffset,
+                                sizeof(v), cudaMemcpyDeviceToHost),
+                     "coverprune_call_stats: copy"));
+  out->gain_evaluations = v[0];
+  out->rounds = v[1];
+  return CP_OK;
 }
 
 int coverprune_cost(const void* feats, int dtype, const float* pos, const int32_t* frame,

@@ -47,6 +47,15 @@ static_assert(sizeof(SceneStats) == 64, "SceneStats layout");
 
 constexpr double kRangeEps = 1e-6;
 
+// Layout of the 256-byte status block at the start of every workspace
+// (zeroed at the start of every call):
+//   int32 [0]      status word (cp_status of the first device-side error)
+//   int32 [4..7]   diagnostics of a CP_EDEVICE (step, scene, block, index)
+//   uint32 [16]    barrier self-test counter (byte 64)
+//   uint64 [16..17] (bytes 128..143) SGS gain evaluations and rounds
+constexpr size_t kStatusBytes = 256;
+constexpr size_t kCallStatsOffset = 128;
+
 // Device attributes cached per device.
 struct DeviceInfo {
   int sm_count;

@@ -148,6 +148,7 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
   const int gw = c * SGS_WARPS + w, nw = cps * SGS_WARPS;
   const size_t nscenes = gridDim.x / cps;
   bool alive = true;
+  unsigned long long my_evals = 0ull;  // rows this warp evaluated (lane 0 counts)
   for (int step = 0; step < K && alive; ++step) {
     unsigned long long best = 0ull;
     for (int t = gw; t < N; t += nw) {
@@ -156,6 +157,7 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
           LOCAL ? local_row_gain(Sb + (size_t)t * P.g, NB + (size_t)t * P.kk, t, P.g, sm_m, sm_v,
                                  lane)
                 : dense_row_gain(Cb + (size_t)t * ldc, sm_m, sm_v, ncols, lane);
+      ++my_evals;
       const unsigned long long key = gain_key(acc, t);
       best = key > best ? key : best;
     }
@@ -223,6 +225,10 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
     __syncthreads();
   }
 
+  unsigned long long* cstats = reinterpret_cast<unsigned long long*>(
+      reinterpret_cast<unsigned char*>(status) + kCallStatsOffset);
+  if (lane == 0 && my_evals) atomicAdd(&cstats[0], my_evals);
+  if (c == 0 && threadIdx.x == 0) atomicAdd(&cstats[1], (unsigned long long)K);
   if (c == 0 && alive && objective) {
     const double F = objective_sum(sm_m, sm_v, N);
     if (threadIdx.x == 0) objective[b] = F;
@@ -314,6 +320,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
   uint32_t* fresh = chosen + nwords;                            // [nwords]
   __shared__ unsigned long long s_wkey[LZ_WARPS];
   __shared__ int s_wfresh[LZ_WARPS];
+  unsigned long long my_evals = 0ull, my_rounds = 0ull;  // lane 0 / thread 0 count
 
   const int b = blockIdx.x;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -338,6 +345,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
   for (int t = w; t < N; t += LZ_WARPS) {
     const float g0 = gain_of(t);
     if (lane == 0) ub[t] = g0;
+    ++my_evals;
   }
   const int S = (N + LZ_WARPS - 1) / LZ_WARPS;
   const int t_lo = w * S, t_hi = min(N, t_lo + S);
@@ -347,6 +355,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
     __syncthreads();
     int pick = -1;
     for (int round = 0; round <= N; ++round) {
+      ++my_rounds;
       unsigned long long best = 0ull;
       for (int t = t_lo + lane; t < t_hi; t += 32)
         if (!(chosen[t >> 5] & (1u << (t & 31)))) {
@@ -377,6 +386,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
       if (!mine_fresh && mine > BF) {  // this slice's best might still win
         const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
         const float g = gain_of(t);
+        ++my_evals;
         if (lane == 0) {
           ub[t] = g;
           atomicOr(&fresh[t >> 5], 1u << (t & 31));
@@ -416,6 +426,10 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
     __syncthreads();
   }
 
+  unsigned long long* cstats = reinterpret_cast<unsigned long long*>(
+      reinterpret_cast<unsigned char*>(status) + kCallStatsOffset);
+  if (lane == 0 && my_evals) atomicAdd(&cstats[0], my_evals);
+  if (threadIdx.x == 0) atomicAdd(&cstats[1], my_rounds);
   if (objective) {
     const double F = objective_sum(sm_m, sm_v, N);
     if (threadIdx.x == 0) objective[b] = F;
