@@ -52,6 +52,28 @@ def make_batch(seeds):
         return pool.map(_gen, seeds)
 
 
+def rank_seeds(rank: int, per_rank: int = SCENES) -> list:
+    """Scene seeds of one rank: every rank prunes its own scenes (weak
+    scaling across scenes, no collective on the data path)."""
+    return list(range(rank * per_rank, rank * per_rank + per_rank))
+
+
+def reduce_max(x: float, dist, device) -> float:
+    """Max of a per-rank number over all ranks (identity without a process
+    group): the whole job lasts as long as its slowest rank."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(scenes_per_rank: int, world: int, ms_max: float) -> float:
+    """Scenes per second of the whole job."""
+    return scenes_per_rank * world / (ms_max / 1000.0)
+
+
 def measured_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -250,11 +272,7 @@ def run_ours(args, rank, world, local_rank, raw):
         torch.cuda.synchronize()
 
     def max_over_ranks(x):
-        if dist is None:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return reduce_max(x, dist, dev)
 
     for _ in range(args.warmup):
         step()
@@ -276,7 +294,7 @@ def run_ours(args, rank, world, local_rank, raw):
     if st != cp.CP_OK:
         raise RuntimeError(f"device status after the timed region: {cp.status_string(st)}")
     ms_step = max_over_ranks(ev0.elapsed_time(ev1) / args.steps)
-    value = B * world / (ms_step / 1000.0)
+    value = whole_job_rate(B, world, ms_step)
 
     # roofline of the SGS kernel from its own events and its counted reads:
     # every gain evaluation reads one padded cost row, every step one row
@@ -497,7 +515,7 @@ def main():
         run_reference(args, rank, world)
         return
     # scenes are drawn in a spawned pool before any CUDA use
-    raw = make_batch(list(range(rank * SCENES, rank * SCENES + SCENES)))
+    raw = make_batch(rank_seeds(rank))
     run_ours(args, rank, world, local_rank, raw)
 
 
