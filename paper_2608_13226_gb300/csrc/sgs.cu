@@ -44,41 +44,60 @@ __device__ __forceinline__ float gain_term(float acc, float v, float m, float c)
   return __fmaf_rn(v, fmaxf(__fsub_rn(m, c), 0.0f), acc);
 }
 
-// gain(t) over a dense padded row (ncols % 4 == 0, pad v = 0).  Lane l sums
-// the float4 chunks l, l+32, l+64, ... in ascending order, then a butterfly:
-// the same fixed order in every kernel that evaluates a gain.  The result is
-// identical in all lanes.
-__device__ __forceinline__ float dense_row_gain(const float* __restrict__ crow,
-                                                const float* sm_m, const float* sm_v, int ncols,
-                                                int lane) {
+// Partial gain over quarter q of a dense padded row (ncols % 4 == 0, pad
+// v = 0): the row's float4 chunks are cut into four contiguous quarters;
+// lane l sums chunks l, l+32, ... of the quarter in ascending order, then a
+// butterfly (identical result in every lane).
+__device__ __forceinline__ float quarter_gain(const float* __restrict__ crow, const float* sm_m,
+                                              const float* sm_v, int ncols, int q, int lane) {
   const float4* row = reinterpret_cast<const float4*>(crow);
   const float4* m4 = reinterpret_cast<const float4*>(sm_m);
   const float4* v4 = reinterpret_cast<const float4*>(sm_v);
   const int nq = ncols >> 2;
+  const int Q4 = (nq + 3) >> 2;
+  const int q_end = min(nq, (q + 1) * Q4);
   float acc = 0.0f;
-  int q = lane;
-  for (; q + 224 < nq; q += 256) {
+  int i = q * Q4 + lane;
+  for (; i + 224 < q_end; i += 256) {
     float4 cs[8];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) cs[u] = ld_stream_f4(row + q + 32 * u);
+    for (int u = 0; u < 8; ++u) cs[u] = ld_stream_f4(row + i + 32 * u);
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
-      const float4 mm = m4[q + 32 * u], vv = v4[q + 32 * u];
+      const float4 mm = m4[i + 32 * u], vv = v4[i + 32 * u];
       acc = gain_term(acc, vv.x, mm.x, cs[u].x);
       acc = gain_term(acc, vv.y, mm.y, cs[u].y);
       acc = gain_term(acc, vv.z, mm.z, cs[u].z);
       acc = gain_term(acc, vv.w, mm.w, cs[u].w);
     }
   }
-  for (; q < nq; q += 32) {
-    const float4 c0 = ld_stream_f4(row + q);
-    const float4 mm = m4[q], vv = v4[q];
+  for (; i < q_end; i += 32) {
+    const float4 c0 = ld_stream_f4(row + i);
+    const float4 mm = m4[i], vv = v4[i];
     acc = gain_term(acc, vv.x, mm.x, c0.x);
     acc = gain_term(acc, vv.y, mm.y, c0.y);
     acc = gain_term(acc, vv.z, mm.z, c0.z);
     acc = gain_term(acc, vv.w, mm.w, c0.w);
   }
   return warp_sum(acc);
+}
+
+// The four quarter sums combined in one fixed order.
+__device__ __forceinline__ float combine_quarters(float s0, float s1, float s2, float s3) {
+  return __fadd_rn(__fadd_rn(__fadd_rn(s0, s1), s2), s3);
+}
+
+// gain(t) over a dense padded row, by one warp: the same quarters and the
+// same combination as the four-warp evaluation of the lazy kernel, so every
+// kernel computes bit-identical gains.
+__device__ __forceinline__ float dense_row_gain(const float* __restrict__ crow,
+                                                const float* sm_m, const float* sm_v, int ncols,
+                                                int lane) {
+  const float s0 = quarter_gain(crow, sm_m, sm_v, ncols, 0, lane);
+  const float s1 = quarter_gain(crow, sm_m, sm_v, ncols, 1, lane);
+  const float s2 = quarter_gain(crow, sm_m, sm_v, ncols, 2, lane);
+  const float s3 = quarter_gain(crow, sm_m, sm_v, ncols, 3, lane);
+  return combine_quarters(s0, s1, s2, s3);
 }
 
 // gain(t) over the local neighbourhood M_g(t): slab row of g costs, member
@@ -436,6 +455,304 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Dense lazy SGS on a thread-block cluster.  The C blocks of a cluster share
+// one scene: block c owns the candidates [c*NC, (c+1)*NC) and keeps its own
+// copy of the scene's (m, v); its 32 warps form 8 quads, each owning a slice
+// of the block's candidates.  A round: every quad scans its slice for the
+// best bound; the C*8 quad bests are exchanged through distributed shared
+// memory after a cluster barrier; if the largest is exact (fresh) it is the
+// step's winner, otherwise every quad whose stale best could still win
+// re-evaluates it, one quarter of the row per warp (quarters combined in the
+// fixed order of dense_row_gain, so the gains are bit-identical to the full
+// sweep's).  The winner's row then lowers every block's copy of m.
+//
+// The round barrier is a monotone arrival counter in block 0's shared
+// memory (release add, acquire spin bounded by the call's time limit; no
+// phase can alias).  The quad bests are double-buffered by round parity, so
+// one barrier per round suffices.  Errors never return early: every block
+// reaches the final hardware cluster barrier, after which no block touches
+// another's shared memory.
+// ---------------------------------------------------------------------------
+constexpr int QD_QUADS = LZ_WARPS / 4;
+
+__device__ __forceinline__ void quad_sync(int k) {
+  asm volatile("bar.sync %0, 128;" ::"r"(1 + k) : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ unsigned long long ld_dsmem_u64(uint32_t a) {
+  unsigned long long v;
+  asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_dsmem_u32(uint32_t a) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_acquire_dsmem_u32(uint32_t a) {
+  uint32_t v;
+  asm volatile("ld.acquire.cluster.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_dsmem_add(uint32_t a, uint32_t v) {
+  asm volatile("red.release.cluster.shared::cluster.add.u32 [%0], %1;" ::"r"(a), "r"(v)
+               : "memory");
+}
+__device__ __forceinline__ void hw_cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+
+__global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(
+    const float* __restrict__ cost, int64_t ldc, const float* __restrict__ v_all, DevParams P,
+    int N, int K, int C, int32_t* __restrict__ order32, float* __restrict__ gains,
+    double* __restrict__ objective, int* status) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int ncols = (int)ldc;
+  const int NC = (N + C - 1) / C;                 // candidates per block
+  const int nwords = (NC + 31) >> 5;
+  float* sm_m = reinterpret_cast<float*>(smem);   // [ncols] coverage cost (full copy)
+  float* sm_v = sm_m + ncols;                     // [ncols] capacity
+  float* ub = sm_v + ncols;                       // [NC] last computed gain, own candidates
+  uint32_t* chosen = reinterpret_cast<uint32_t*>(ub + NC);  // [nwords] own candidates
+  uint32_t* fresh = chosen + nwords;                        // [nwords]
+  __shared__ unsigned long long s_wq[LZ_WARPS];
+  __shared__ unsigned long long s_key[2][QD_QUADS];  // by round parity, read by the cluster
+  __shared__ uint32_t s_fresh[2][QD_QUADS];
+  __shared__ float s_part[QD_QUADS][4];
+  __shared__ unsigned long long s_G, s_BF;
+  __shared__ uint32_t s_ctr;                      // round barrier counter (used in block 0)
+  __shared__ int s_ok;
+
+  const uint32_t crank = cluster_ctarank();
+  const int b = blockIdx.x / C;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int k = w >> 2, q = w & 3, tq = threadIdx.x & 127;
+  const int c0 = (int)crank * NC;                 // first candidate of this block
+  const int nown = max(0, min(N, c0 + NC) - c0);  // own candidates
+  const float* v = v_all + (size_t)b * N;
+  const float* Cb = cost + (size_t)b * N * ldc;
+  unsigned long long my_evals = 0ull, my_rounds = 0ull;
+  const uint32_t ctr0 = map_rank(smem_addr(&s_ctr), 0);
+
+  for (int j = threadIdx.x; j < ncols; j += LZ_THREADS) {
+    sm_m[j] = j < N ? P.m0 : 0.0f;
+    sm_v[j] = j < N ? v[j] : 0.0f;
+  }
+  for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) chosen[i] = 0u;
+  if (threadIdx.x == 0) s_ctr = 0u;
+  hw_cluster_sync();  // every block initialised before anyone arrives on block 0
+
+  // step 0: every own candidate's gain exactly, one warp per row
+  for (int t = w; t < nown; t += LZ_WARPS) {
+    const float g0 = dense_row_gain(Cb + (size_t)(c0 + t) * ldc, sm_m, sm_v, ncols, lane);
+    if (lane == 0) ub[t] = g0;
+    ++my_evals;
+  }
+  const int S = (nown + QD_QUADS - 1) / QD_QUADS;
+  const int t_lo = k * S, t_hi = min(nown, t_lo + S);  // quad slice, own indices
+  uint32_t gr = 0;  // rounds so far (all blocks count alike)
+  bool ok = true;
+
+  for (int step = 0; step < K && ok; ++step) {
+    for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) fresh[i] = step == 0 ? ~0u : 0u;
+    __syncthreads();
+    int pick = -1;
+    for (int round = 0; round <= N && ok; ++round, ++gr) {
+      ++my_rounds;
+      const int par = gr & 1;
+      unsigned long long best = 0ull;
+      for (int t = t_lo + tq; t < t_hi; t += 128)
+        if (!(chosen[t >> 5] & (1u << (t & 31)))) {
+          const unsigned long long key = gain_key(ub[t], c0 + t);
+          best = key > best ? key : best;
+        }
+      best = warp_max_u64(best);
+      if (lane == 0) s_wq[w] = best;
+      quad_sync(k);
+      if (q == 0 && lane == 0) {
+        unsigned long long kb = s_wq[4 * k];
+        for (int i = 1; i < 4; ++i) kb = s_wq[4 * k + i] > kb ? s_wq[4 * k + i] : kb;
+        const int bt = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull)) - c0;
+        s_key[par][k] = kb;
+        s_fresh[par][k] = kb != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
+      }
+      // cluster round barrier: arrive on block 0's counter, wait for C * (gr+1)
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        int good = 1;
+        red_release_dsmem_add(ctr0, 1u);
+        const uint32_t target = (gr + 1u) * (uint32_t)C;
+        const uint64_t t0 = globaltimer_ns();
+        uint32_t spins = 0;
+        while (ld_acquire_dsmem_u32(ctr0) < target) {
+          if ((++spins & 63u) == 0) {
+            if (ld_volatile_i32(status) != 0) { good = 0; break; }
+            if (globaltimer_ns() - t0 > P.timeout_ns) {
+              set_status(status, CP_ETIMEOUT);
+              good = 0;
+              break;
+            }
+          }
+        }
+        s_ok = good;
+      }
+      __syncthreads();
+      if (!s_ok) {
+        ok = false;
+        break;
+      }
+      if (w == 0) {  // gather the cluster's quad bests
+        unsigned long long G = 0ull, BF = 0ull;
+        (void)ld_acquire_dsmem_u32(ctr0);  // this lane's own acquire of the round
+        for (int e = lane; e < C * QD_QUADS; e += 32) {
+          const uint32_t r = (uint32_t)(e / QD_QUADS), kk = (uint32_t)(e % QD_QUADS);
+          const unsigned long long key = ld_dsmem_u64(map_rank(smem_addr(&s_key[par][kk]), r));
+          const uint32_t fr = ld_dsmem_u32(map_rank(smem_addr(&s_fresh[par][kk]), r));
+          G = key > G ? key : G;
+          if (fr) BF = key > BF ? key : BF;
+        }
+        G = warp_max_u64(G);
+        BF = warp_max_u64(BF);
+        if (lane == 0) {
+          s_G = G;
+          s_BF = BF;
+        }
+      }
+      __syncthreads();
+      const unsigned long long G = s_G, BF = s_BF;
+      if (G != 0ull && G == BF) {  // the largest bound is exact: the winner
+        pick = (int)(0xFFFFFFFFu - (uint32_t)(G & 0xFFFFFFFFull));
+        ++gr;
+        break;
+      }
+      if (G == 0ull) {  // no candidate left (never for K <= N)
+        ++gr;
+        break;
+      }
+      const unsigned long long mine = s_key[par][k];
+      if (!s_fresh[par][k] && mine > BF) {  // this quad's best might still win
+        const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
+        const float part = quarter_gain(Cb + (size_t)t * ldc, sm_m, sm_v, ncols, q, lane);
+        if (lane == 0) s_part[k][q] = part;
+        quad_sync(k);
+        if (q == 0 && lane == 0) {
+          const int tl = t - c0;
+          ub[tl] = combine_quarters(s_part[k][0], s_part[k][1], s_part[k][2], s_part[k][3]);
+          atomicOr(&fresh[tl >> 5], 1u << (tl & 31));  // quads may share a word
+          ++my_evals;
+        }
+      }
+      __syncthreads();
+    }
+    if (!ok) break;
+    const bool bad = pick < 0 || pick >= N ||
+                     (pick >= c0 && pick < c0 + nown &&
+                      (chosen[(pick - c0) >> 5] & (1u << ((pick - c0) & 31))) != 0u);
+    __syncthreads();
+    if (bad) {  // never expected; cluster-uniform
+      if (threadIdx.x == 0 && crank == 0 && atomicCAS(status, 0, CP_EDEVICE) == 0) {
+        status[4] = step;
+        status[5] = b;
+        status[6] = (int)crank;
+        status[7] = pick;
+      }
+      ok = false;
+      break;
+    }
+    if (threadIdx.x == 0) {
+      if (pick >= c0 && pick < c0 + nown) chosen[(pick - c0) >> 5] |= 1u << ((pick - c0) & 31);
+      if (crank == 0) {
+        order32[(size_t)b * K + step] = pick;
+        if (gains) gains[(size_t)b * K + step] = __uint_as_float((uint32_t)(s_G >> 32));
+      }
+    }
+    // S <- S u {t*} (Eq. sgs_update), on this block's copy of m
+    const float* row = Cb + (size_t)pick * ldc;
+    for (int j = threadIdx.x; j < N; j += LZ_THREADS) sm_m[j] = fminf(sm_m[j], __ldg(row + j));
+    __syncthreads();
+  }
+
+  unsigned long long* cstats = reinterpret_cast<unsigned long long*>(
+      reinterpret_cast<unsigned char*>(status) + kCallStatsOffset);
+  if (lane == 0 && my_evals) atomicAdd(&cstats[0], my_evals);
+  if (threadIdx.x == 0 && crank == 0) atomicAdd(&cstats[1], my_rounds);
+  if (ok && crank == 0 && objective) {
+    const double F = objective_sum(sm_m, sm_v, N);
+    if (threadIdx.x == 0) objective[b] = F;
+  }
+  hw_cluster_sync();  // nobody leaves while a peer may still read its shared memory
+}
+
+// Blocks per scene for the cluster kernel: the largest power of two <= 8
+// such that every scene's cluster can be resident at once.
+static int cluster_size_for(int64_t B, int sm_count) {
+  int C = 8;
+  while (C > 1 && (int64_t)C * B > sm_count) C >>= 1;
+  return C;
+}
+
+static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* v,
+                                   const DevParams& P, int64_t B, int64_t N, int64_t K,
+                                   int32_t* order32, float* gains, double* objective, int* status,
+                                   cudaStream_t s) {
+  DeviceInfo di;
+  if (device_info(&di) != CP_OK) return CP_ECUDA;
+  auto fn = k_sgs_lazy_cl;
+  for (int C = cluster_size_for(B, di.sm_count); C >= 1; C >>= 1) {
+    const int64_t NC = (N + C - 1) / C;
+    const size_t smem = sizeof(float) * (size_t)(2 * ldc + NC) +
+                        2 * sizeof(uint32_t) * (size_t)((NC + 31) / 32);
+    if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem),
+                    "launch_sgs_lazy_cluster: smem attribute") != CP_OK)
+      return CP_ECUDA;
+    if (C > 8 &&
+        cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1),
+                    "launch_sgs_lazy_cluster: cluster attribute") != CP_OK)
+      return CP_ECUDA;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(B * C));
+    cfg.blockDim = dim3(LZ_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&clusters, (const void*)fn, &cfg) != cudaSuccess ||
+        clusters < 1) {
+      (void)cudaGetLastError();
+      continue;  // this cluster shape cannot be resident: try a smaller one
+    }
+    int Ni = (int)N, Ki = (int)K;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, fn, cost, ldc, v, P, Ni, Ki, C, order32, gains,
+                                       objective, status);
+    note_launch();
+    return cuda_status(e, "launch_sgs_lazy_cluster");
+  }
+  note_message("launch_sgs_lazy_cluster: no resident cluster shape");
+  return CP_EUNSUPPORTED;
+}
+
 template <bool LOCAL>
 static int sgs_lazy_launch(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                            const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
@@ -444,7 +761,9 @@ static int sgs_lazy_launch(const float* cost, int64_t ldc, const float* slab, co
   const int64_t ncols = LOCAL ? N : ldc;
   const size_t smem = sizeof(float) * (size_t)(2 * ncols + N) +
                       2 * sizeof(uint32_t) * (size_t)((N + 31) / 32);
-  auto fn = k_sgs_lazy<LOCAL>;
+  if (!LOCAL)
+    return sgs_lazy_cluster_launch(cost, ldc, v, P, B, N, K, order32, gains, objective, status, s);
+  auto fn = k_sgs_lazy<true>;
   if (smem > 48 * 1024 &&
       cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
                   "launch_sgs_lazy: smem attribute") != CP_OK)
