@@ -61,9 +61,11 @@ def main():
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1))
     st = cp.coverprune_check(ws)
-    print(json.dumps({"scene": a.scene, "op": a.op, "batch": a.batch, "N": cfg.N, "D": cfg.D,
-                      "K": K, "g": a.g, "ms_median": statistics.median(times),
-                      "status": cp.status_string(st)}))
+    line = {"scene": a.scene, "op": a.op, "batch": a.batch, "N": cfg.N, "D": cfg.D, "K": K,
+            "g": a.g, "ms_median": statistics.median(times), "status": cp.status_string(st)}
+    if a.op == "select":
+        line["call_stats"] = cp.coverprune_call_stats(ws)
+    print(json.dumps(line))
     if st != cp.CP_OK:
         raise SystemExit(1)
 
