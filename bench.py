@@ -297,24 +297,26 @@ def run_ours(args, rank, world, local_rank, raw):
     value = whole_job_rate(B, world, ms_step)
 
     # roofline of the SGS kernel from its own events and its counted reads:
-    # every gain evaluation reads one padded cost row, every step one row
-    # to update the coverage cost
+    # the cost bytes its gain evaluations read (the kernel counts them: row
+    # blocks known to hold only zero terms are skipped) plus one row per
+    # step to update the coverage cost
     hbm, tf_burst, tf_sust, peak_kind = measured_peaks()
     cstats = cp.coverprune_call_stats(ws)
     sgs_ms, sgs_launches = prof["sgs"]
     launches_per_step = max(sgs_launches // args.steps, 1)
     ldc = (N + 3) // 4 * 4
-    sgs_bytes_per_step = cstats["gain_evaluations"] * ldc * 4 + B * K * N * 4
+    sgs_bytes_per_step = cstats["cost_bytes_read"] + B * K * N * 4
     sgs_launch_ms = sgs_ms / max(sgs_launches, 1)
     sgs_gbs = (sgs_bytes_per_step / launches_per_step) / (sgs_launch_ms / 1000.0) / 1e9
     roofline_sgs = {"bound": "hbm", "kernel": "k_sgs_lazy<dense>", "achieved": round(sgs_gbs, 1),
                     "peak": hbm, "unit": "GB/s", "frac": round(sgs_gbs / hbm, 4),
-                    "traffic": read_traffic("k_sgs_lazy", cstats["gain_evaluations"]),
+                    "traffic": read_traffic("k_sgs_lazy", sgs_bytes_per_step // launches_per_step),
                     "peak_source": peak_kind,
                     "algorithmic_bytes_per_launch": sgs_bytes_per_step // launches_per_step,
                     "avg_launch_ms": round(sgs_launch_ms, 3),
                     "gain_evaluations_per_step": cstats["gain_evaluations"],
                     "rounds_per_step": cstats["rounds"],
+                    "cost_bytes_read_per_step": cstats["cost_bytes_read"],
                     "full_sweep_evaluations_per_step": B * (K * N - K * (K - 1) // 2)}
     def tflops(stage, flops_per_call):
         ms, launches = prof[stage]
@@ -359,11 +361,11 @@ def run_ours(args, rank, world, local_rank, raw):
     fprof = cp.coverprune_profile_read()
     fstats = cp.coverprune_call_stats(ws)
     f_ms = fprof["sgs"][0] / max(fprof["sgs"][1], 1)
-    f_bytes = fstats["gain_evaluations"] * ldc * 4 + B * K * N * 4
+    f_bytes = fstats["cost_bytes_read"] + B * K * N * 4
     f_gbs = f_bytes / (f_ms / 1000.0) / 1e9
     sweep = {"bound": "hbm", "kernel": "k_sgs<dense>", "achieved": round(f_gbs, 1), "peak": hbm,
              "unit": "GB/s", "frac": round(f_gbs / hbm, 4),
-             "traffic": read_traffic("k_sgs", fstats["gain_evaluations"]),
+             "traffic": read_traffic("k_sgs", f_bytes),
              "algorithmic_bytes_per_launch": f_bytes, "avg_launch_ms": round(f_ms, 3)}
     stages = {k: round(v[0] / args.steps, 3) for k, v in prof.items() if v[0] > 0}
     gpu_launches = sum(v[1] for v in prof.values())
@@ -478,12 +480,12 @@ def run_ours(args, rank, world, local_rank, raw):
         dist.destroy_process_group()
 
 
-def read_traffic(kernel: str, evaluations: int):
+def read_traffic(kernel: str, algorithmic_bytes: int):
     """DRAM bytes of one SGS launch, scaled from the committed ncu record of
-    that kernel (profiles/<kernel>_traffic.txt: bytes per gain evaluation,
-    which reads one cost row) by the launch's evaluations; None when no
-    record exists or the kernel source has changed since the counters were
-    taken."""
+    that kernel (profiles/<kernel>_traffic.txt: its DRAM bytes per
+    algorithmic byte on a captured launch) by this launch's algorithmic
+    bytes; None when no record exists or the kernel source has changed
+    since the counters were taken."""
     import hashlib
     path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
     try:
@@ -496,7 +498,7 @@ def read_traffic(kernel: str, evaluations: int):
                        for f in ("sgs.cu", "common.cuh"))
         if hashlib.sha256(src).hexdigest()[:16] != rec.get("source_sha256"):
             return None
-        return float(rec["traffic_bytes_per_evaluation"]) * evaluations
+        return round(float(rec["dram_bytes_per_algorithmic_byte"]) * algorithmic_bytes)
     except (OSError, KeyError, ValueError):
         return None
 

@@ -328,11 +328,16 @@ int coverprune_profile_read(double* ms, int64_t* launches, int n);
  *                     local slab (g floats)
  *   rounds            decision rounds over all scenes and steps (lazy mode:
  *                     a step needs one or more; full sweep: one per step)
+ *   cost_bytes_read   bytes of cost rows (or slab rows and their neighbour
+ *                     indices) the gain evaluations read; the dense lazy
+ *                     kernel skips row blocks whose terms are known to be
+ *                     zero, so this can be well below gain_evaluations * 4N
  * Returns CP_OK, CP_EINVAL or CP_ECUDA.
  */
 typedef struct {
   uint64_t gain_evaluations;
   uint64_t rounds;
+  uint64_t cost_bytes_read;
 } cp_call_stats;
 int coverprune_call_stats(const void* ws, cp_stream_t stream, cp_call_stats* out);
 

@@ -51,7 +51,8 @@ class _CpParams(C.Structure):
 
 
 class _CallStats(C.Structure):
-    _fields_ = [("gain_evaluations", C.c_uint64), ("rounds", C.c_uint64)]
+    _fields_ = [("gain_evaluations", C.c_uint64), ("rounds", C.c_uint64),
+                ("cost_bytes_read", C.c_uint64)]
 
 
 @dataclass
@@ -380,11 +381,13 @@ def coverprune_profile_read() -> dict:
 
 
 def coverprune_call_stats(ws) -> dict:
-    """{"gain_evaluations", "rounds"} of the last coverprune_select on ws."""
+    """{"gain_evaluations", "rounds", "cost_bytes_read"} of the last
+    coverprune_select on ws."""
     out = _CallStats()
     _check(_lib().coverprune_call_stats(_ptr(ws), _stream(), C.byref(out)),
            "coverprune_call_stats")
-    return {"gain_evaluations": int(out.gain_evaluations), "rounds": int(out.rounds)}
+    return {"gain_evaluations": int(out.gain_evaluations), "rounds": int(out.rounds),
+            "cost_bytes_read": int(out.cost_bytes_read)}
 
 
 def coverprune_version() -> int:

@@ -372,12 +372,13 @@ int coverprune_check(const void* ws, cp_stream_t stream) {
 int coverprune_call_stats(const void* ws, cp_stream_t stream, cp_call_stats* out) {
   if (!ws || !out) return CP_EINVAL;
   CP_TRY(cuda_status(cudaStreamSynchronize((cudaStream_t)stream), "coverprune_call_stats: stream"));
-  unsigned long long v[2] = {0, 0};
+  unsigned long long v[3] = {0, 0, 0};
   CP_TRY(cuda_status(cudaMemcpy(v, static_cast<const unsigned char*>(ws) + kCallStatsOffset,
                                 sizeof(v), cudaMemcpyDeviceToHost),
                      "coverprune_call_stats: copy"));
   out->gain_evaluations = v[0];
   out->rounds = v[1];
+  out->cost_bytes_read = v[2];
   return CP_OK;
 }
 

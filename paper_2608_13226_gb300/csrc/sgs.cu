@@ -87,6 +87,71 @@ __device__ __forceinline__ float combine_quarters(float s0, float s1, float s2, 
   return __fadd_rn(__fadd_rn(__fadd_rn(s0, s1), s2), s3);
 }
 
+// quarter_gain over the blocks a mask names.  Quarter q's float4 chunks are
+// visited in iterations of 32 (iteration u: chunks q*Q4 + 32u + lane); bit
+// u >> bit_shift of m16 says whether iteration u may hold a positive term.  An
+// iteration whose terms are all zero leaves every lane's sum unchanged (each
+// term is v * max(m - C, 0) = +0 and acc + 0 = acc), so skipping it returns
+// exactly quarter_gain's value.  A term stays zero once m <= C, because m
+// only decreases; out16 gets the bits of the iterations that still have
+// some m > C.  Up to 8 needed iterations are loaded before any is summed.
+__device__ __forceinline__ float quarter_gain_masked(const float* __restrict__ crow,
+                                                     const float* sm_m, const float* sm_v,
+                                                     int ncols, int q, int lane, uint32_t m16,
+                                                     int bit_shift, uint32_t& out16, int& nread) {
+  const float4* row = reinterpret_cast<const float4*>(crow);
+  const float4* m4 = reinterpret_cast<const float4*>(sm_m);
+  const float4* v4 = reinterpret_cast<const float4*>(sm_v);
+  const int nq = ncols >> 2;
+  const int Q4 = (nq + 3) >> 2;
+  const int q0 = q * Q4;
+  const int q_end = min(nq, q0 + Q4);
+  const int nit = q_end > q0 ? (q_end - q0 + 31) >> 5 : 0;
+  uint32_t todo = m16 & 0xFFFFu;
+  if (bit_shift) {  // each bit covers two iterations: spread bit i to bits 2i, 2i+1
+    todo = (todo | (todo << 8)) & 0x00FF00FFu;
+    todo = (todo | (todo << 4)) & 0x0F0F0F0Fu;
+    todo = (todo | (todo << 2)) & 0x33333333u;
+    todo = (todo | (todo << 1)) & 0x55555555u;
+    todo |= todo << 1;
+  }
+  if (nit < 32) todo &= (1u << nit) - 1u;
+  nread = __popc(todo);
+  float acc = 0.0f;
+  uint32_t nzb = 0u;
+  while (todo) {
+    int us[8];
+#pragma unroll
+    for (int s = 0; s < 8; ++s) {
+      us[s] = todo ? __ffs(todo) - 1 : -1;
+      todo &= todo - 1u;
+    }
+    float4 cs[8];
+#pragma unroll
+    for (int s = 0; s < 8; ++s) {
+      const int i = q0 + 32 * us[s] + lane;
+      cs[s] = (us[s] >= 0 && i < q_end) ? ld_stream_f4(row + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int s = 0; s < 8; ++s) {
+      if (us[s] < 0) break;  // warp-uniform
+      const int i = q0 + 32 * us[s] + lane;
+      bool nz = false;
+      if (i < q_end) {
+        const float4 mm = m4[i], vv = v4[i];
+        acc = gain_term(acc, vv.x, mm.x, cs[s].x);
+        acc = gain_term(acc, vv.y, mm.y, cs[s].y);
+        acc = gain_term(acc, vv.z, mm.z, cs[s].z);
+        acc = gain_term(acc, vv.w, mm.w, cs[s].w);
+        nz = (mm.x > cs[s].x) | (mm.y > cs[s].y) | (mm.z > cs[s].z) | (mm.w > cs[s].w);
+      }
+      if (__any_sync(0xFFFFFFFFu, nz)) nzb |= 1u << (us[s] >> bit_shift);
+    }
+  }
+  out16 = nzb;
+  return warp_sum(acc);
+}
+
 // gain(t) over a dense padded row, by one warp: the same quarters and the
 // same combination as the four-warp evaluation of the lazy kernel, so every
 // kernel computes bit-identical gains.
@@ -248,6 +313,8 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
       reinterpret_cast<unsigned char*>(status) + kCallStatsOffset);
   if (lane == 0 && my_evals) atomicAdd(&cstats[0], my_evals);
   if (c == 0 && threadIdx.x == 0) atomicAdd(&cstats[1], (unsigned long long)K);
+  if (lane == 0 && my_evals)
+    atomicAdd(&cstats[2], my_evals * (unsigned long long)(LOCAL ? 8 * P.g : 4 * ldc));
   if (c == 0 && alive && objective) {
     const double F = objective_sum(sm_m, sm_v, N);
     if (threadIdx.x == 0) objective[b] = F;
@@ -449,6 +516,8 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
       reinterpret_cast<unsigned char*>(status) + kCallStatsOffset);
   if (lane == 0 && my_evals) atomicAdd(&cstats[0], my_evals);
   if (threadIdx.x == 0) atomicAdd(&cstats[1], my_rounds);
+  if (lane == 0 && my_evals)
+    atomicAdd(&cstats[2], my_evals * (unsigned long long)(LOCAL ? 8 * P.g : 4 * ldc));
   if (objective) {
     const double F = objective_sum(sm_m, sm_v, N);
     if (threadIdx.x == 0) objective[b] = F;
@@ -458,24 +527,40 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
 
 // ---------------------------------------------------------------------------
 // Dense lazy SGS on a thread-block cluster.  The C blocks of a cluster share
-// one scene: block c owns the candidates [c*NC, (c+1)*NC) and keeps its own
-// copy of the scene's (m, v); its 32 warps form 8 quads, each owning a slice
-// of the block's candidates.  A round: every quad scans its slice for the
-// best bound; the C*8 quad bests are exchanged through distributed shared
-// memory after a cluster barrier; if the largest is exact (fresh) it is the
-// step's winner, otherwise every quad whose stale best could still win
-// re-evaluates it, one quarter of the row per warp (quarters combined in the
-// fixed order of dense_row_gain, so the gains are bit-identical to the full
-// sweep's).  The winner's row then lowers every block's copy of m.
+// one scene: block c owns the candidates t = c (mod C) and keeps its own
+// copy of the scene's (m, v); its 32 warps form 8 quads, quad k owning the
+// block's candidates of own index k (mod 8).  Interleaving spreads tokens
+// with nearby indices -- in a scene they are nearby in space, so one pick
+// lowers their gains together -- over all quads of the cluster, which then
+// re-evaluate them in the same round.  A step has two phases.
 //
-// The round barrier is a monotone arrival counter in block 0's shared
-// memory (release add, acquire spin bounded by the call's time limit; no
-// phase can alias).  The quad bests are double-buffered by round parity, so
-// one barrier per round suffices.  Errors never return early: every block
-// reaches the final hardware cluster barrier, after which no block touches
-// another's shared memory.
+//  1. Local certification, with block barriers only.  Each round every quad
+//     finds the best key of its slice.  If the block's largest key is exact
+//     ("fresh") it is the block's result r_c; if it is below the cluster's
+//     hint h (the largest exact key any block has computed this step) the
+//     block cannot hold the winner and r_c is its best fresh key; otherwise
+//     every quad whose stale best could still win re-evaluates it, one
+//     quarter of the row per warp (quarters combined in the fixed order of
+//     dense_row_gain, so gains are bit-identical to the full sweep's).  A
+//     new exact key is pushed into every block's hint: a max over keys
+//     tagged with the step, so a late push from an earlier step never wins.
+//     Each own candidate keeps a 64-bit mask of the row blocks that held a
+//     positive term at its last evaluation (when the masks fit in shared
+//     memory); an evaluation reads only those blocks (quarter_gain_masked).
+//  2. Exchange.  Block c stores r_c into its slot in every block and adds to
+//     that block's arrival counter (release); every block waits on its own
+//     counter (acquire, bounded) and takes the largest result.
+//
+// The largest result is the step's winner: every key of block c is at most
+// r_c or below a hint, and the block that computed a hint reports a result
+// at least as large; so max_c r_c bounds every candidate's key and is itself
+// an exact key.  Slots and counters are double-buffered by step parity (a
+// block can be at most one step ahead of a peer's exchange).  Errors never
+// return early: every block reaches the final hardware cluster barrier,
+// after which no block touches another's shared memory.
 // ---------------------------------------------------------------------------
 constexpr int QD_QUADS = LZ_WARPS / 4;
+constexpr int CL_MAX = 8;  // blocks per cluster (portable cluster size)
 
 __device__ __forceinline__ void quad_sync(int k) {
   asm volatile("bar.sync %0, 128;" ::"r"(1 + k) : "memory");
@@ -493,15 +578,8 @@ __device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
   return r;
 }
-__device__ __forceinline__ unsigned long long ld_dsmem_u64(uint32_t a) {
-  unsigned long long v;
-  asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");
-  return v;
-}
-__device__ __forceinline__ uint32_t ld_dsmem_u32(uint32_t a) {
-  uint32_t v;
-  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
-  return v;
+__device__ __forceinline__ void st_dsmem_u64(uint32_t a, unsigned long long v) {
+  asm volatile("st.shared::cluster.u64 [%0], %1;" ::"r"(a), "l"(v) : "memory");
 }
 __device__ __forceinline__ uint32_t ld_acquire_dsmem_u32(uint32_t a) {
   uint32_t v;
@@ -512,190 +590,346 @@ __device__ __forceinline__ void red_release_dsmem_add(uint32_t a, uint32_t v) {
   asm volatile("red.release.cluster.shared::cluster.add.u32 [%0], %1;" ::"r"(a), "r"(v)
                : "memory");
 }
+__device__ __forceinline__ void red_dsmem_max_u64(uint32_t a, unsigned long long v) {
+  asm volatile("red.relaxed.cluster.shared::cluster.max.u64 [%0], %1;" ::"r"(a), "l"(v)
+               : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_volatile_u64(const unsigned long long* p) {
+  return *reinterpret_cast<const volatile unsigned long long*>(p);
+}
 __device__ __forceinline__ void hw_cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
                    : "memory");
 }
 
-__global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(
-    const float* __restrict__ cost, int64_t ldc, const float* __restrict__ v_all, DevParams P,
-    int N, int K, int C, int32_t* __restrict__ order32, float* __restrict__ gains,
-    double* __restrict__ objective, int* status) {
+// Hint format: step in bits 45.., gain bits in 14..44, 16383 - index in
+// 0..13 (N <= 16384 and K <= N): a later step's hint is always larger.
+__device__ __forceinline__ unsigned long long tag_key(unsigned long long key, int step) {
+  const uint32_t t = 0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull);
+  return ((unsigned long long)step << 45) | ((key >> 32) << 14) | (16383u - t);
+}
+__device__ __forceinline__ unsigned long long untag_key(unsigned long long h, int step) {
+  if ((int)(h >> 45) != step || h == 0ull) return 0ull;
+  const uint32_t t = 16383u - (uint32_t)(h & 0x3FFFull);
+  return (((h >> 14) & 0x7FFFFFFFull) << 32) | (0xFFFFFFFFu - t);
+}
+
+// Launch arguments of k_sgs_lazy_cl, precomputed on the host and read from
+// the parameter space (the kernel runs at 64 registers a thread).
+struct LzClArgs {
+  const float* cost;   // [B][N][ldc]
+  const float* v;      // [B][N]
+  int32_t* order32;    // [B][K]
+  float* gains;        // [B][K] or null
+  double* objective;   // [B] or null
+  int* status;
+  int64_t ldc;
+  uint64_t timeout_ns;
+  float m0;
+  int N, K;
+  int C, lgC;          // blocks per cluster, a power of two, and its log2
+  int NC;              // candidates per block, ceil(N / C)
+  int nwords;          // words of a candidate bitmap, ceil(NC / 32)
+  int use_mask;        // block masks kept in shared memory
+  int bit_shift;       // log2 of the quarter iterations per mask bit (0 or 1)
+  uint32_t off_v, off_ub, off_chosen, off_fresh, off_nzm;  // dynamic smem offsets
+};
+
+__global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_constant__ LzClArgs a) {
   extern __shared__ __align__(16) unsigned char smem[];
-  const int ncols = (int)ldc;
-  const int NC = (N + C - 1) / C;                 // candidates per block
-  const int nwords = (NC + 31) >> 5;
-  float* sm_m = reinterpret_cast<float*>(smem);   // [ncols] coverage cost (full copy)
-  float* sm_v = sm_m + ncols;                     // [ncols] capacity
-  float* ub = sm_v + ncols;                       // [NC] last computed gain, own candidates
-  uint32_t* chosen = reinterpret_cast<uint32_t*>(ub + NC);  // [nwords] own candidates
-  uint32_t* fresh = chosen + nwords;                        // [nwords]
-  __shared__ unsigned long long s_wq[LZ_WARPS];
-  __shared__ unsigned long long s_key[2][QD_QUADS];  // by round parity, read by the cluster
-  __shared__ uint32_t s_fresh[2][QD_QUADS];
+  float* sm_m = reinterpret_cast<float*>(smem);                    // [ldc] coverage cost
+  float* sm_v = reinterpret_cast<float*>(smem + a.off_v);          // [ldc] capacity
+  float* ub = reinterpret_cast<float*>(smem + a.off_ub);           // [NC] last computed gain
+  uint32_t* chosen = reinterpret_cast<uint32_t*>(smem + a.off_chosen);  // [nwords]
+  uint32_t* fresh = reinterpret_cast<uint32_t*>(smem + a.off_fresh);    // [nwords]
+  uint16_t* nzm = reinterpret_cast<uint16_t*>(smem + a.off_nzm);   // [NC][4] if use_mask
+  __shared__ unsigned long long s_wq[LZ_WARPS];    // best key of each warp's candidates
+  __shared__ unsigned long long s_qkey[QD_QUADS];  // best key of each quad
+  __shared__ uint32_t s_qfresh[QD_QUADS];
   __shared__ float s_part[QD_QUADS][4];
-  __shared__ unsigned long long s_G, s_BF;
-  __shared__ uint32_t s_ctr;                      // round barrier counter (used in block 0)
+  __shared__ unsigned long long s_G[2], s_BF[2];   // largest key / largest fresh key, by round parity
+  __shared__ uint32_t s_dirty[2];                  // warps to rescan, by round parity
+  __shared__ unsigned long long s_hint;            // tagged; pushed by every block
+  __shared__ unsigned long long s_H;               // this round's hint, untagged
+  __shared__ unsigned long long s_res[2][CL_MAX];  // exchange: results, by step parity
+  __shared__ unsigned long long s_resm[2][CL_MAX];  // exchange: their block masks
+  __shared__ uint32_t s_cnt[2];                    // exchange arrivals, by step parity
+  __shared__ unsigned long long s_W, s_WM;
+  __shared__ unsigned long long s_stats[3];        // evaluations, rounds, cost bytes read
   __shared__ int s_ok;
 
+  const int ncols = (int)a.ldc;
+  const int lgC = a.lgC;
   const uint32_t crank = cluster_ctarank();
-  const int b = blockIdx.x / C;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int k = w >> 2, q = w & 3, tq = threadIdx.x & 127;
-  const int c0 = (int)crank * NC;                 // first candidate of this block
-  const int nown = max(0, min(N, c0 + NC) - c0);  // own candidates
-  const float* v = v_all + (size_t)b * N;
-  const float* Cb = cost + (size_t)b * N * ldc;
-  unsigned long long my_evals = 0ull, my_rounds = 0ull;
-  const uint32_t ctr0 = map_rank(smem_addr(&s_ctr), 0);
+  const int k = w >> 2, q = w & 3;
+  // own index tl <-> candidate t = (tl << lgC) | crank; quad k scans the own
+  // indices k + 8 * (threadIdx.x & 127) + 1024 i, so warp 4k + ((tl >> 8) & 3)
+  // holds tl
+  const int nown = a.N > (int)crank ? (a.N - (int)crank + a.C - 1) >> lgC : 0;
+  const float* Cb = a.cost + (size_t)(blockIdx.x >> lgC) * a.N * a.ldc;
 
-  for (int j = threadIdx.x; j < ncols; j += LZ_THREADS) {
-    sm_m[j] = j < N ? P.m0 : 0.0f;
-    sm_v[j] = j < N ? v[j] : 0.0f;
+  {
+    const float* v = a.v + (size_t)(blockIdx.x >> lgC) * a.N;
+    for (int j = threadIdx.x; j < ncols; j += LZ_THREADS) {
+      sm_m[j] = j < a.N ? a.m0 : 0.0f;
+      sm_v[j] = j < a.N ? v[j] : 0.0f;
+    }
   }
-  for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) chosen[i] = 0u;
-  if (threadIdx.x == 0) s_ctr = 0u;
-  hw_cluster_sync();  // every block initialised before anyone arrives on block 0
+  for (int i = threadIdx.x; i < a.nwords; i += LZ_THREADS) {
+    chosen[i] = 0u;
+    fresh[i] = ~0u;  // step 0: every gain below is exact
+  }
+  if (threadIdx.x < 3) s_stats[threadIdx.x] = 0ull;
+  if (threadIdx.x == 0) {
+    s_hint = 0ull;
+    s_cnt[0] = s_cnt[1] = 0u;
+    s_G[0] = s_G[1] = s_BF[0] = s_BF[1] = 0ull;
+    s_dirty[0] = 0xFFFFFFFFu;  // the first round scans everything
+    s_dirty[1] = 0u;
+  }
+  hw_cluster_sync();  // every block initialised before any peer writes to it
 
   // step 0: every own candidate's gain exactly, one warp per row
-  for (int t = w; t < nown; t += LZ_WARPS) {
-    const float g0 = dense_row_gain(Cb + (size_t)(c0 + t) * ldc, sm_m, sm_v, ncols, lane);
-    if (lane == 0) ub[t] = g0;
-    ++my_evals;
+  for (int tl = w; tl < nown; tl += LZ_WARPS) {
+    const float* crow = Cb + (size_t)((tl << lgC) | (int)crank) * a.ldc;
+    float g0;
+    if (a.use_mask) {
+      // combine_quarters is the left fold ((s0 + s1) + s2) + s3
+      int nr_all = 0;
+      g0 = 0.0f;
+#pragma unroll 1
+      for (int qq = 0; qq < 4; ++qq) {
+        uint32_t o;
+        int nr;
+        const float sq =
+            quarter_gain_masked(crow, sm_m, sm_v, ncols, qq, lane, 0xFFFFu, a.bit_shift, o, nr);
+        g0 = qq == 0 ? sq : __fadd_rn(g0, sq);
+        if (lane == 0) nzm[4 * tl + qq] = (uint16_t)o;
+        nr_all += nr;
+      }
+      if (lane == 0) atomicAdd(&s_stats[2], 512ull * (unsigned long long)nr_all);
+    } else {
+      g0 = dense_row_gain(crow, sm_m, sm_v, ncols, lane);
+      if (lane == 0) atomicAdd(&s_stats[2], 4ull * (unsigned long long)ncols);
+    }
+    if (lane == 0) {
+      ub[tl] = g0;
+      atomicAdd(&s_stats[0], 1ull);
+    }
   }
-  const int S = (nown + QD_QUADS - 1) / QD_QUADS;
-  const int t_lo = k * S, t_hi = min(nown, t_lo + S);  // quad slice, own indices
-  uint32_t gr = 0;  // rounds so far (all blocks count alike)
   bool ok = true;
+  uint32_t gr = 0;  // rounds of this block so far (every thread alike)
 
-  for (int step = 0; step < K && ok; ++step) {
-    for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) fresh[i] = step == 0 ? ~0u : 0u;
+  for (int step = 0; step < a.K && ok; ++step) {
+    if (step > 0)
+      for (int i = threadIdx.x; i < a.nwords; i += LZ_THREADS) fresh[i] = 0u;
     __syncthreads();
-    int pick = -1;
-    for (int round = 0; round <= N && ok; ++round, ++gr) {
-      ++my_rounds;
+
+    // ---- phase 1: this block's result
+    unsigned long long R = 0ull;
+    for (int round = 0; round <= a.NC; ++round) {
       const int par = gr & 1;
-      unsigned long long best = 0ull;
-      for (int t = t_lo + tq; t < t_hi; t += 128)
-        if (!(chosen[t >> 5] & (1u << (t & 31)))) {
-          const unsigned long long key = gain_key(ub[t], c0 + t);
-          best = key > best ? key : best;
-        }
-      best = warp_max_u64(best);
-      if (lane == 0) s_wq[w] = best;
+      ++gr;
+      if ((s_dirty[par] >> w) & 1u) {  // this warp's candidates changed: rescan them
+        unsigned long long best = 0ull;
+        for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128)
+          if (!(chosen[tl >> 5] & (1u << (tl & 31)))) {
+            const unsigned long long key = gain_key(ub[tl], (tl << lgC) | (int)crank);
+            best = key > best ? key : best;
+          }
+        best = warp_max_u64(best);
+        if (lane == 0) s_wq[w] = best;
+      }
+      if (threadIdx.x == 0) {
+        s_H = untag_key(ld_volatile_u64(&s_hint), step);
+        ++s_stats[1];
+        s_dirty[par ^ 1] = 0u;  // the next round's slots
+        s_G[par ^ 1] = 0ull;
+        s_BF[par ^ 1] = 0ull;
+      }
       quad_sync(k);
       if (q == 0 && lane == 0) {
         unsigned long long kb = s_wq[4 * k];
         for (int i = 1; i < 4; ++i) kb = s_wq[4 * k + i] > kb ? s_wq[4 * k + i] : kb;
-        const int bt = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull)) - c0;
-        s_key[par][k] = kb;
-        s_fresh[par][k] = kb != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
+        const int bt = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull)) >> lgC;
+        const uint32_t fr = kb != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
+        s_qkey[k] = kb;
+        s_qfresh[k] = fr;
+        atomicMax(&s_G[par], kb);
+        if (fr) atomicMax(&s_BF[par], kb);
       }
-      // cluster round barrier: arrive on block 0's counter, wait for C * (gr+1)
       __syncthreads();
-      if (threadIdx.x == 0) {
+      const unsigned long long G = s_G[par], BF = s_BF[par], H = s_H;
+      if (G == 0ull) break;  // no candidate left in this block
+      if (G == BF) {         // the block's largest bound is exact
+        R = G;
+        break;
+      }
+      if (G < H) {  // nothing here can beat an exact key of another block
+        R = BF;
+        break;
+      }
+      const unsigned long long mine = s_qkey[k];
+      const unsigned long long floor_key = BF > H ? BF : H;
+      if (!s_qfresh[k] && mine > floor_key) {  // this quad's best might still win
+        const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
+        const int tl = t >> lgC;
+        float part;
+        if (a.use_mask) {
+          uint32_t o;
+          int nr;
+          part = quarter_gain_masked(Cb + (size_t)t * a.ldc, sm_m, sm_v, ncols, q, lane,
+                                     nzm[4 * tl + q], a.bit_shift, o, nr);
+          if (lane == 0) {
+            nzm[4 * tl + q] = (uint16_t)o;
+            atomicAdd(&s_stats[2], 512ull * (unsigned long long)nr);
+          }
+        } else {
+          part = quarter_gain(Cb + (size_t)t * a.ldc, sm_m, sm_v, ncols, q, lane);
+          if (lane == 0) atomicAdd(&s_stats[2], (unsigned long long)ncols);  // a quarter row
+        }
+        if (lane == 0) s_part[k][q] = part;
+        quad_sync(k);
+        if (q == 0 && lane == 0) {
+          const float g = combine_quarters(s_part[k][0], s_part[k][1], s_part[k][2], s_part[k][3]);
+          ub[tl] = g;
+          atomicOr(&fresh[tl >> 5], 1u << (tl & 31));  // quads may share a word
+          atomicOr(&s_dirty[par ^ 1], 1u << (4 * k + ((tl >> 8) & 3)));
+          atomicAdd(&s_stats[0], 1ull);
+          const unsigned long long nk = gain_key(g, t);
+          if (nk > floor_key) {  // a new best exact key: tell the cluster
+            const unsigned long long tagged = tag_key(nk, step);
+            for (int r = 0; r < a.C; ++r)
+              red_dsmem_max_u64(map_rank(smem_addr(&s_hint), r), tagged);
+          }
+        }
+      }
+      __syncthreads();
+    }
+
+    // ---- phase 2: exchange the C results with their block masks
+    const int par = step & 1;
+    if (w == 0) {
+      if (lane < a.C) {
+        unsigned long long RM = R == 0ull ? 0ull : ~0ull;
+        if (R != 0ull && a.use_mask) {
+          const int tl = (int)(0xFFFFFFFFu - (uint32_t)(R & 0xFFFFFFFFull)) >> lgC;
+          RM = (unsigned long long)nzm[4 * tl] | ((unsigned long long)nzm[4 * tl + 1] << 16) |
+               ((unsigned long long)nzm[4 * tl + 2] << 32) |
+               ((unsigned long long)nzm[4 * tl + 3] << 48);
+        }
+        st_dsmem_u64(map_rank(smem_addr(&s_res[par][crank]), lane), R);
+        st_dsmem_u64(map_rank(smem_addr(&s_resm[par][crank]), lane), RM);
+        red_release_dsmem_add(map_rank(smem_addr(&s_cnt[par]), lane), 1u);
+      }
+      if (lane == 0) {
         int good = 1;
-        red_release_dsmem_add(ctr0, 1u);
-        const uint32_t target = (gr + 1u) * (uint32_t)C;
-        const uint64_t t0 = globaltimer_ns();
+        const uint32_t own_cnt = map_rank(smem_addr(&s_cnt[par]), crank);
+        const uint32_t target = (uint32_t)a.C * (uint32_t)((step >> 1) + 1);
+        uint64_t t0 = 0;  // read the clock only once the wait is not short
         uint32_t spins = 0;
-        while (ld_acquire_dsmem_u32(ctr0) < target) {
+        while (ld_acquire_dsmem_u32(own_cnt) < target) {
           if ((++spins & 63u) == 0) {
-            if (ld_volatile_i32(status) != 0) { good = 0; break; }
-            if (globaltimer_ns() - t0 > P.timeout_ns) {
-              set_status(status, CP_ETIMEOUT);
+            if (ld_volatile_i32(a.status) != 0) { good = 0; break; }
+            if (t0 == 0) {
+              t0 = globaltimer_ns();
+            } else if (globaltimer_ns() - t0 > a.timeout_ns) {
+              set_status(a.status, CP_ETIMEOUT);
               good = 0;
               break;
             }
           }
         }
+        unsigned long long W = 0ull, WM = 0ull;
+        if (good)
+          for (int r = 0; r < a.C; ++r) {
+            const unsigned long long x = ld_volatile_u64(&s_res[par][r]);
+            if (x > W) {
+              W = x;
+              WM = ld_volatile_u64(&s_resm[par][r]);
+            }
+          }
+        s_W = W;
+        s_WM = WM;
         s_ok = good;
       }
-      __syncthreads();
-      if (!s_ok) {
-        ok = false;
-        break;
-      }
-      if (w == 0) {  // gather the cluster's quad bests
-        unsigned long long G = 0ull, BF = 0ull;
-        (void)ld_acquire_dsmem_u32(ctr0);  // this lane's own acquire of the round
-        for (int e = lane; e < C * QD_QUADS; e += 32) {
-          const uint32_t r = (uint32_t)(e / QD_QUADS), kk = (uint32_t)(e % QD_QUADS);
-          const unsigned long long key = ld_dsmem_u64(map_rank(smem_addr(&s_key[par][kk]), r));
-          const uint32_t fr = ld_dsmem_u32(map_rank(smem_addr(&s_fresh[par][kk]), r));
-          G = key > G ? key : G;
-          if (fr) BF = key > BF ? key : BF;
-        }
-        G = warp_max_u64(G);
-        BF = warp_max_u64(BF);
-        if (lane == 0) {
-          s_G = G;
-          s_BF = BF;
-        }
-      }
-      __syncthreads();
-      const unsigned long long G = s_G, BF = s_BF;
-      if (G != 0ull && G == BF) {  // the largest bound is exact: the winner
-        pick = (int)(0xFFFFFFFFu - (uint32_t)(G & 0xFFFFFFFFull));
-        ++gr;
-        break;
-      }
-      if (G == 0ull) {  // no candidate left (never for K <= N)
-        ++gr;
-        break;
-      }
-      const unsigned long long mine = s_key[par][k];
-      if (!s_fresh[par][k] && mine > BF) {  // this quad's best might still win
-        const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
-        const float part = quarter_gain(Cb + (size_t)t * ldc, sm_m, sm_v, ncols, q, lane);
-        if (lane == 0) s_part[k][q] = part;
-        quad_sync(k);
-        if (q == 0 && lane == 0) {
-          const int tl = t - c0;
-          ub[tl] = combine_quarters(s_part[k][0], s_part[k][1], s_part[k][2], s_part[k][3]);
-          atomicOr(&fresh[tl >> 5], 1u << (tl & 31));  // quads may share a word
-          ++my_evals;
-        }
-      }
-      __syncthreads();
     }
-    if (!ok) break;
-    const bool bad = pick < 0 || pick >= N ||
-                     (pick >= c0 && pick < c0 + nown &&
-                      (chosen[(pick - c0) >> 5] & (1u << ((pick - c0) & 31))) != 0u);
     __syncthreads();
-    if (bad) {  // never expected; cluster-uniform
-      if (threadIdx.x == 0 && crank == 0 && atomicCAS(status, 0, CP_EDEVICE) == 0) {
-        status[4] = step;
-        status[5] = b;
-        status[6] = (int)crank;
-        status[7] = pick;
+    if (!s_ok) {
+      ok = false;
+      break;
+    }
+    const unsigned long long W = s_W, WM = s_WM;
+    const int pick = W == 0ull ? -1 : (int)(0xFFFFFFFFu - (uint32_t)(W & 0xFFFFFFFFull));
+    const bool own = pick >= 0 && (pick & (a.C - 1)) == (int)crank;
+    const int ptl = pick >> lgC;
+    const bool bad = pick < 0 || pick >= a.N ||
+                     (own && (chosen[ptl >> 5] & (1u << (ptl & 31))) != 0u);
+    __syncthreads();
+    if (bad) {  // never expected
+      if (threadIdx.x == 0 && atomicCAS(a.status, 0, CP_EDEVICE) == 0) {
+        a.status[4] = step;
+        a.status[5] = (int)(blockIdx.x >> lgC);
+        a.status[6] = (int)crank;
+        a.status[7] = pick;
       }
       ok = false;
       break;
     }
     if (threadIdx.x == 0) {
-      if (pick >= c0 && pick < c0 + nown) chosen[(pick - c0) >> 5] |= 1u << ((pick - c0) & 31);
+      if (own) {
+        chosen[ptl >> 5] |= 1u << (ptl & 31);
+        s_dirty[gr & 1] |= 1u << (4 * (ptl & 7) + ((ptl >> 8) & 3));  // its warp rescans
+      }
       if (crank == 0) {
-        order32[(size_t)b * K + step] = pick;
-        if (gains) gains[(size_t)b * K + step] = __uint_as_float((uint32_t)(s_G >> 32));
+        const size_t o = (size_t)(blockIdx.x >> lgC) * a.K + step;
+        a.order32[o] = pick;
+        if (a.gains) a.gains[o] = __uint_as_float((uint32_t)(W >> 32));
       }
     }
-    // S <- S u {t*} (Eq. sgs_update), on this block's copy of m
-    const float* row = Cb + (size_t)pick * ldc;
-    for (int j = threadIdx.x; j < N; j += LZ_THREADS) sm_m[j] = fminf(sm_m[j], __ldg(row + j));
+    // S <- S u {t*} (Eq. sgs_update), on this block's copy of m.  Only the
+    // row blocks of the winner's mask can lower m: the winner was evaluated
+    // at the current m, and a block outside its mask has m <= C throughout.
+    // Pad columns hold C = 0 and m = 0, so whole float4 chunks are safe.
+    {
+      const float4* row = reinterpret_cast<const float4*>(Cb + (size_t)pick * a.ldc);
+      float4* m4 = reinterpret_cast<float4*>(sm_m);
+      const int nq = ncols >> 2, Q4 = (nq + 3) >> 2;
+      for (int bb = w; bb < 64; bb += LZ_WARPS) {
+        if (!((WM >> bb) & 1ull)) continue;
+        const int q0 = (bb >> 4) * Q4, q_end = min(nq, q0 + Q4);
+        const int u0 = (bb & 15) << a.bit_shift, u1 = ((bb & 15) + 1) << a.bit_shift;
+        for (int u = u0; u < u1; ++u) {
+          const int i = q0 + 32 * u + lane;
+          if (i < q_end) {
+            const float4 c = __ldg(row + i);
+            float4 mm = m4[i];
+            mm.x = fminf(mm.x, c.x);
+            mm.y = fminf(mm.y, c.y);
+            mm.z = fminf(mm.z, c.z);
+            mm.w = fminf(mm.w, c.w);
+            m4[i] = mm;
+          }
+        }
+      }
+    }
     __syncthreads();
   }
 
   unsigned long long* cstats = reinterpret_cast<unsigned long long*>(
-      reinterpret_cast<unsigned char*>(status) + kCallStatsOffset);
-  if (lane == 0 && my_evals) atomicAdd(&cstats[0], my_evals);
-  if (threadIdx.x == 0 && crank == 0) atomicAdd(&cstats[1], my_rounds);
-  if (ok && crank == 0 && objective) {
-    const double F = objective_sum(sm_m, sm_v, N);
-    if (threadIdx.x == 0) objective[b] = F;
+      reinterpret_cast<unsigned char*>(a.status) + kCallStatsOffset);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    atomicAdd(&cstats[0], s_stats[0]);
+    if (crank == 0) atomicAdd(&cstats[1], s_stats[1]);
+    atomicAdd(&cstats[2], s_stats[2]);
   }
-  hw_cluster_sync();  // nobody leaves while a peer may still read its shared memory
+  if (ok && crank == 0 && a.objective) {
+    const double F = objective_sum(sm_m, sm_v, a.N);
+    if (threadIdx.x == 0) a.objective[blockIdx.x >> lgC] = F;
+  }
+  hw_cluster_sync();  // nobody leaves while a peer may still write to its shared memory
 }
 
 // Blocks per scene for the cluster kernel: the largest power of two <= 8
@@ -714,16 +948,37 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
   if (device_info(&di) != CP_OK) return CP_ECUDA;
   auto fn = k_sgs_lazy_cl;
   for (int C = cluster_size_for(B, di.sm_count); C >= 1; C >>= 1) {
-    const int64_t NC = (N + C - 1) / C;
-    const size_t smem = sizeof(float) * (size_t)(2 * ldc + NC) +
-                        2 * sizeof(uint32_t) * (size_t)((NC + 31) / 32);
+    LzClArgs a{};
+    a.cost = cost;
+    a.v = v;
+    a.order32 = order32;
+    a.gains = gains;
+    a.objective = objective;
+    a.status = status;
+    a.ldc = ldc;
+    a.timeout_ns = P.timeout_ns;
+    a.m0 = P.m0;
+    a.N = (int)N;
+    a.K = (int)K;
+    a.C = C;
+    a.lgC = C >= 8 ? 3 : C >= 4 ? 2 : C >= 2 ? 1 : 0;
+    a.NC = (int)((N + C - 1) / C);
+    a.nwords = (a.NC + 31) / 32;
+    const int nit_max = (int)(((ldc / 4 + 3) / 4 + 31) / 32);  // iterations per quarter
+    a.bit_shift = nit_max <= 16 ? 0 : 1;
+    a.off_v = (uint32_t)(sizeof(float) * ldc);
+    a.off_ub = (uint32_t)(sizeof(float) * 2 * ldc);
+    a.off_chosen = a.off_ub + (uint32_t)(sizeof(float) * a.NC);
+    a.off_fresh = a.off_chosen + (uint32_t)(sizeof(uint32_t) * a.nwords);
+    a.off_nzm = a.off_fresh + (uint32_t)(sizeof(uint32_t) * a.nwords);
+    const size_t smem_plain = a.off_nzm;
+    const size_t smem_mask = smem_plain + 4 * sizeof(uint16_t) * (size_t)a.NC;
+    // the block masks live in shared memory when they fit beside (m, v)
+    a.use_mask = smem_mask + 2048 <= (size_t)di.max_smem_optin ? 1 : 0;
+    const size_t smem = a.use_mask ? smem_mask : smem_plain;
     if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem),
                     "launch_sgs_lazy_cluster: smem attribute") != CP_OK)
-      return CP_ECUDA;
-    if (C > 8 &&
-        cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1),
-                    "launch_sgs_lazy_cluster: cluster attribute") != CP_OK)
       return CP_ECUDA;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(B * C));
@@ -743,9 +998,7 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
       (void)cudaGetLastError();
       continue;  // this cluster shape cannot be resident: try a smaller one
     }
-    int Ni = (int)N, Ki = (int)K;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, fn, cost, ldc, v, P, Ni, Ki, C, order32, gains,
-                                       objective, status);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, fn, a);
     note_launch();
     return cuda_status(e, "launch_sgs_lazy_cluster");
   }
