@@ -139,11 +139,18 @@ __device__ __forceinline__ float quarter_gain_masked(const float* __restrict__ c
       bool nz = false;
       if (i < q_end) {
         const float4 mm = m4[i], vv = v4[i];
-        acc = gain_term(acc, vv.x, mm.x, cs[s].x);
-        acc = gain_term(acc, vv.y, mm.y, cs[s].y);
-        acc = gain_term(acc, vv.z, mm.z, cs[s].z);
-        acc = gain_term(acc, vv.w, mm.w, cs[s].w);
-        nz = (mm.x > cs[s].x) | (mm.y > cs[s].y) | (mm.z > cs[s].z) | (mm.w > cs[s].w);
+        // d = max(m - C, 0) is +0 or positive, so the OR of the bit
+        // patterns is zero iff all four terms are zero
+        const float d0 = fmaxf(__fsub_rn(mm.x, cs[s].x), 0.0f);
+        const float d1 = fmaxf(__fsub_rn(mm.y, cs[s].y), 0.0f);
+        const float d2 = fmaxf(__fsub_rn(mm.z, cs[s].z), 0.0f);
+        const float d3 = fmaxf(__fsub_rn(mm.w, cs[s].w), 0.0f);
+        acc = __fmaf_rn(vv.x, d0, acc);
+        acc = __fmaf_rn(vv.y, d1, acc);
+        acc = __fmaf_rn(vv.z, d2, acc);
+        acc = __fmaf_rn(vv.w, d3, acc);
+        nz = (__float_as_uint(d0) | __float_as_uint(d1) | __float_as_uint(d2) |
+              __float_as_uint(d3)) != 0u;
       }
       if (__any_sync(0xFFFFFFFFu, nz)) nzb |= 1u << (us[s] >> bit_shift);
     }
@@ -597,6 +604,9 @@ __device__ __forceinline__ void red_dsmem_max_u64(uint32_t a, unsigned long long
 __device__ __forceinline__ unsigned long long ld_volatile_u64(const unsigned long long* p) {
   return *reinterpret_cast<const volatile unsigned long long*>(p);
 }
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
 __device__ __forceinline__ void hw_cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
                    : "memory");
@@ -645,18 +655,18 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   uint16_t* nzm = reinterpret_cast<uint16_t*>(smem + a.off_nzm);   // [NC][4] if use_mask
   __shared__ unsigned long long s_wq[LZ_WARPS];    // best key of each warp's candidates
   __shared__ unsigned long long s_qkey[QD_QUADS];  // best key of each quad
-  __shared__ uint32_t s_qfresh[QD_QUADS];
+  __shared__ uint32_t s_qfresh[QD_QUADS];          // ... and whether it is exact
   __shared__ float s_part[QD_QUADS][4];
-  __shared__ unsigned long long s_G[2], s_BF[2];   // largest key / largest fresh key, by round parity
-  __shared__ uint32_t s_dirty[2];                  // warps to rescan, by round parity
+  __shared__ unsigned long long s_G[3], s_BF[3];   // block's largest key / largest exact
+                                                   // key, one slot per round (mod 3)
   __shared__ unsigned long long s_hint;            // tagged; pushed by every block
-  __shared__ unsigned long long s_H;               // this round's hint, untagged
+  __shared__ unsigned long long s_H;               // the hint for the next decision
   __shared__ unsigned long long s_res[2][CL_MAX];  // exchange: results, by step parity
   __shared__ unsigned long long s_resm[2][CL_MAX];  // exchange: their block masks
   __shared__ uint32_t s_cnt[2];                    // exchange arrivals, by step parity
   __shared__ unsigned long long s_W, s_WM;
   __shared__ unsigned long long s_stats[3];        // evaluations, rounds, cost bytes read
-  __shared__ int s_ok;
+  __shared__ int s_ok;                             // 1 ok, 0 stop, 2 inconsistent winner
 
   const int ncols = (int)a.ldc;
   const int lgC = a.lgC;
@@ -664,8 +674,8 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int k = w >> 2, q = w & 3;
   // own index tl <-> candidate t = (tl << lgC) | crank; quad k scans the own
-  // indices k + 8 * (threadIdx.x & 127) + 1024 i, so warp 4k + ((tl >> 8) & 3)
-  // holds tl
+  // indices k + 8 * (threadIdx.x & 127) + 1024 i, so warp 4 * (tl & 7) +
+  // ((tl >> 8) & 3) holds tl
   const int nown = a.N > (int)crank ? (a.N - (int)crank + a.C - 1) >> lgC : 0;
   const float* Cb = a.cost + (size_t)(blockIdx.x >> lgC) * a.N * a.ldc;
 
@@ -680,13 +690,14 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     chosen[i] = 0u;
     fresh[i] = ~0u;  // step 0: every gain below is exact
   }
-  if (threadIdx.x < 3) s_stats[threadIdx.x] = 0ull;
+  if (threadIdx.x < 3) {
+    s_stats[threadIdx.x] = 0ull;
+    s_G[threadIdx.x] = 0ull;
+    s_BF[threadIdx.x] = 0ull;
+  }
   if (threadIdx.x == 0) {
     s_hint = 0ull;
     s_cnt[0] = s_cnt[1] = 0u;
-    s_G[0] = s_G[1] = s_BF[0] = s_BF[1] = 0ull;
-    s_dirty[0] = 0xFFFFFFFFu;  // the first round scans everything
-    s_dirty[1] = 0u;
   }
   hw_cluster_sync();  // every block initialised before any peer writes to it
 
@@ -718,49 +729,62 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
       atomicAdd(&s_stats[0], 1ull);
     }
   }
+  __syncthreads();
+
+  // the best key of this warp's remaining candidates, into s_wq[w]
+  auto warp_rescan = [&]() {
+    unsigned long long best = 0ull;
+    for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128)
+      if (!(chosen[tl >> 5] & (1u << (tl & 31)))) {
+        const unsigned long long key = gain_key(ub[tl], (tl << lgC) | (int)crank);
+        best = key > best ? key : best;
+      }
+    best = warp_max_u64(best);
+    if (lane == 0) s_wq[w] = best;
+  };
+  // quad leader: the quad's best key and whether it is exact (all_stale:
+  // at the start of a step after the first, without reading the bitmap,
+  // whose reset by other warps is not yet ordered before this read)
+  auto quad_best = [&](bool all_stale) -> unsigned long long {
+    unsigned long long kb = s_wq[4 * k];
+    for (int i = 1; i < 4; ++i) kb = s_wq[4 * k + i] > kb ? s_wq[4 * k + i] : kb;
+    const int bt = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull)) >> lgC;
+    s_qkey[k] = kb;
+    s_qfresh[k] = !all_stale && kb != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
+    return kb;
+  };
+
   bool ok = true;
-  uint32_t gr = 0;  // rounds of this block so far (every thread alike)
+  int slot = 0;  // decision slot of the next round
+  warp_rescan();  // step 0 starts from every warp's best
 
   for (int step = 0; step < a.K && ok; ++step) {
-    if (step > 0)
-      for (int i = threadIdx.x; i < a.nwords; i += LZ_THREADS) fresh[i] = 0u;
+    // ---- step start: the quad bests into the first decision slot (the
+    // warp that held the last pick has rescanned; m is updated, fresh reset)
+    quad_sync(k);
+    if (q == 0 && lane == 0) {
+      const unsigned long long kb = quad_best(step > 0);
+      atomicMax(&s_G[slot], kb);
+      if (s_qfresh[k]) atomicMax(&s_BF[slot], kb);
+    }
+    if (threadIdx.x == 0) s_H = untag_key(ld_volatile_u64(&s_hint), step);
     __syncthreads();
 
-    // ---- phase 1: this block's result
+    // ---- phase 1: this block's result.  A round reads its slot, clears
+    // the slot two rounds ahead (read two rounds ago) and fills the next.
     unsigned long long R = 0ull;
     for (int round = 0; round <= a.NC; ++round) {
-      const int par = gr & 1;
-      ++gr;
-      if ((s_dirty[par] >> w) & 1u) {  // this warp's candidates changed: rescan them
-        unsigned long long best = 0ull;
-        for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128)
-          if (!(chosen[tl >> 5] & (1u << (tl & 31)))) {
-            const unsigned long long key = gain_key(ub[tl], (tl << lgC) | (int)crank);
-            best = key > best ? key : best;
-          }
-        best = warp_max_u64(best);
-        if (lane == 0) s_wq[w] = best;
-      }
+      const unsigned long long G = s_G[slot], BF = s_BF[slot], H = s_H;
+      const unsigned long long mine = s_qkey[k];
+      const uint32_t mine_fresh = s_qfresh[k];
+      const int nslot = slot == 2 ? 0 : slot + 1;
+      const int cslot = nslot == 2 ? 0 : nslot + 1;
       if (threadIdx.x == 0) {
-        s_H = untag_key(ld_volatile_u64(&s_hint), step);
+        s_G[cslot] = 0ull;
+        s_BF[cslot] = 0ull;
         ++s_stats[1];
-        s_dirty[par ^ 1] = 0u;  // the next round's slots
-        s_G[par ^ 1] = 0ull;
-        s_BF[par ^ 1] = 0ull;
       }
-      quad_sync(k);
-      if (q == 0 && lane == 0) {
-        unsigned long long kb = s_wq[4 * k];
-        for (int i = 1; i < 4; ++i) kb = s_wq[4 * k + i] > kb ? s_wq[4 * k + i] : kb;
-        const int bt = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull)) >> lgC;
-        const uint32_t fr = kb != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
-        s_qkey[k] = kb;
-        s_qfresh[k] = fr;
-        atomicMax(&s_G[par], kb);
-        if (fr) atomicMax(&s_BF[par], kb);
-      }
-      __syncthreads();
-      const unsigned long long G = s_G[par], BF = s_BF[par], H = s_H;
+      slot = nslot;
       if (G == 0ull) break;  // no candidate left in this block
       if (G == BF) {         // the block's largest bound is exact
         R = G;
@@ -770,9 +794,8 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
         R = BF;
         break;
       }
-      const unsigned long long mine = s_qkey[k];
       const unsigned long long floor_key = BF > H ? BF : H;
-      if (!s_qfresh[k] && mine > floor_key) {  // this quad's best might still win
+      if (!mine_fresh && mine > floor_key) {  // this quad's best might still win
         const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
         const int tl = t >> lgC;
         float part;
@@ -795,7 +818,6 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
           const float g = combine_quarters(s_part[k][0], s_part[k][1], s_part[k][2], s_part[k][3]);
           ub[tl] = g;
           atomicOr(&fresh[tl >> 5], 1u << (tl & 31));  // quads may share a word
-          atomicOr(&s_dirty[par ^ 1], 1u << (4 * k + ((tl >> 8) & 3)));
           atomicAdd(&s_stats[0], 1ull);
           const unsigned long long nk = gain_key(g, t);
           if (nk > floor_key) {  // a new best exact key: tell the cluster
@@ -804,12 +826,40 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
               red_dsmem_max_u64(map_rank(smem_addr(&s_hint), r), tagged);
           }
         }
+        quad_sync(k);
+        if (w == 4 * k + ((tl >> 8) & 3)) warp_rescan();  // the warp holding t
+        quad_sync(k);
+        if (q == 0 && lane == 0) (void)quad_best(false);
       }
+      if (q == 0 && lane == 0) {  // every quad into the next decision
+        atomicMax(&s_G[slot], s_qkey[k]);
+        if (s_qfresh[k]) atomicMax(&s_BF[slot], s_qkey[k]);
+      }
+      if (threadIdx.x == 0) s_H = untag_key(ld_volatile_u64(&s_hint), step);
       __syncthreads();
     }
 
-    // ---- phase 2: exchange the C results with their block masks
+    // ---- phase 2: exchange the C results with their block masks.  Meanwhile
+    // warp 1 of each quad prefetches into L2 the blocks of the quad's best
+    // candidate, which the next step's first round will most likely
+    // re-evaluate (every bound goes stale with the pick)
     const int par = step & 1;
+    if (q == 1 && a.use_mask) {
+      const unsigned long long kb = s_qkey[k];
+      if (kb != 0ull && kb != R) {
+        const int t = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull));
+        const int tl = t >> lgC;
+        const int nq = ncols >> 2, Q4 = (nq + 3) >> 2;
+        const float4* row = reinterpret_cast<const float4*>(Cb + (size_t)t * a.ldc);
+        for (int bb = lane; bb < 64; bb += 32) {
+          if (!((nzm[4 * tl + (bb >> 4)] >> (bb & 15)) & 1u)) continue;
+          const int q0 = (bb >> 4) * Q4, q_end = min(nq, q0 + Q4);
+          const int i0 = q0 + (32 << a.bit_shift) * (bb & 15);
+          const int i1 = min(q_end, i0 + (32 << a.bit_shift));
+          if (i1 > i0) prefetch_l2(row + i0, (uint32_t)(16 * (i1 - i0)));
+        }
+      }
+    }
     if (w == 0) {
       if (lane < a.C) {
         unsigned long long RM = R == 0ull ? 0ull : ~0ull;
@@ -842,7 +892,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
           }
         }
         unsigned long long W = 0ull, WM = 0ull;
-        if (good)
+        if (good) {
           for (int r = 0; r < a.C; ++r) {
             const unsigned long long x = ld_volatile_u64(&s_res[par][r]);
             if (x > W) {
@@ -850,43 +900,39 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
               WM = ld_volatile_u64(&s_resm[par][r]);
             }
           }
+          // the winner must be a valid candidate that this block, if it owns
+          // it, has not picked before (never expected otherwise)
+          const int pick = W == 0ull ? -1 : (int)(0xFFFFFFFFu - (uint32_t)(W & 0xFFFFFFFFull));
+          const int ptl = pick >> lgC;
+          if (pick < 0 || pick >= a.N ||
+              ((pick & (a.C - 1)) == (int)crank && (chosen[ptl >> 5] & (1u << (ptl & 31))))) {
+            good = 2;
+            if (atomicCAS(a.status, 0, CP_EDEVICE) == 0) {
+              a.status[4] = step;
+              a.status[5] = (int)(blockIdx.x >> lgC);
+              a.status[6] = (int)crank;
+              a.status[7] = pick;
+            }
+          }
+        }
         s_W = W;
         s_WM = WM;
         s_ok = good;
       }
     }
     __syncthreads();
-    if (!s_ok) {
+    if (s_ok != 1) {
       ok = false;
       break;
     }
     const unsigned long long W = s_W, WM = s_WM;
-    const int pick = W == 0ull ? -1 : (int)(0xFFFFFFFFu - (uint32_t)(W & 0xFFFFFFFFull));
-    const bool own = pick >= 0 && (pick & (a.C - 1)) == (int)crank;
+    const int pick = (int)(0xFFFFFFFFu - (uint32_t)(W & 0xFFFFFFFFull));
     const int ptl = pick >> lgC;
-    const bool bad = pick < 0 || pick >= a.N ||
-                     (own && (chosen[ptl >> 5] & (1u << (ptl & 31))) != 0u);
-    __syncthreads();
-    if (bad) {  // never expected
-      if (threadIdx.x == 0 && atomicCAS(a.status, 0, CP_EDEVICE) == 0) {
-        a.status[4] = step;
-        a.status[5] = (int)(blockIdx.x >> lgC);
-        a.status[6] = (int)crank;
-        a.status[7] = pick;
-      }
-      ok = false;
-      break;
-    }
-    if (threadIdx.x == 0) {
-      if (own) {
-        chosen[ptl >> 5] |= 1u << (ptl & 31);
-        s_dirty[gr & 1] |= 1u << (4 * (ptl & 7) + ((ptl >> 8) & 3));  // its warp rescans
-      }
-      if (crank == 0) {
-        const size_t o = (size_t)(blockIdx.x >> lgC) * a.K + step;
-        a.order32[o] = pick;
-        if (a.gains) a.gains[o] = __uint_as_float((uint32_t)(W >> 32));
-      }
+    const bool own = (pick & (a.C - 1)) == (int)crank;
+    if (threadIdx.x == 0 && crank == 0) {
+      const size_t o = (size_t)(blockIdx.x >> lgC) * a.K + step;
+      a.order32[o] = pick;
+      if (a.gains) a.gains[o] = __uint_as_float((uint32_t)(W >> 32));
     }
     // S <- S u {t*} (Eq. sgs_update), on this block's copy of m.  Only the
     // row blocks of the winner's mask can lower m: the winner was evaluated
@@ -914,7 +960,13 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
         }
       }
     }
-    __syncthreads();
+    // every bound goes stale; the warp that held the pick drops it
+    for (int i = threadIdx.x; i < a.nwords; i += LZ_THREADS) fresh[i] = 0u;
+    if (own && w == 4 * (ptl & 7) + ((ptl >> 8) & 3)) {
+      if (lane == 0) chosen[ptl >> 5] |= 1u << (ptl & 31);
+      __syncwarp();
+      warp_rescan();
+    }
   }
 
   unsigned long long* cstats = reinterpret_cast<unsigned long long*>(
