@@ -660,7 +660,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   __shared__ unsigned long long s_G[3], s_BF[3];   // block's largest key / largest exact
                                                    // key, one slot per round (mod 3)
   __shared__ unsigned long long s_hint;            // tagged; pushed by every block
-  __shared__ unsigned long long s_H;               // the hint for the next decision
+  __shared__ unsigned long long s_H[3];            // the hint for each decision slot
   __shared__ unsigned long long s_res[2][CL_MAX];  // exchange: results, by step parity
   __shared__ unsigned long long s_resm[2][CL_MAX];  // exchange: their block masks
   __shared__ uint32_t s_cnt[2];                    // exchange arrivals, by step parity
@@ -767,14 +767,16 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
       atomicMax(&s_G[slot], kb);
       if (s_qfresh[k]) atomicMax(&s_BF[slot], kb);
     }
-    if (threadIdx.x == 0) s_H = untag_key(ld_volatile_u64(&s_hint), step);
+    if (threadIdx.x == 0) s_H[slot] = untag_key(ld_volatile_u64(&s_hint), step);
     __syncthreads();
 
     // ---- phase 1: this block's result.  A round reads its slot, clears
-    // the slot two rounds ahead (read two rounds ago) and fills the next.
+    // the slot two rounds ahead (read two rounds ago) and fills the next;
+    // nothing a round reads is written before the block barrier that ends
+    // it, so every thread takes the same decisions.
     unsigned long long R = 0ull;
     for (int round = 0; round <= a.NC; ++round) {
-      const unsigned long long G = s_G[slot], BF = s_BF[slot], H = s_H;
+      const unsigned long long G = s_G[slot], BF = s_BF[slot], H = s_H[slot];
       const unsigned long long mine = s_qkey[k];
       const uint32_t mine_fresh = s_qfresh[k];
       const int nslot = slot == 2 ? 0 : slot + 1;
@@ -814,17 +816,16 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
         }
         if (lane == 0) s_part[k][q] = part;
         quad_sync(k);
-        if (q == 0 && lane == 0) {
+        if (q == 0) {  // the quad's first warp records the gain
           const float g = combine_quarters(s_part[k][0], s_part[k][1], s_part[k][2], s_part[k][3]);
-          ub[tl] = g;
-          atomicOr(&fresh[tl >> 5], 1u << (tl & 31));  // quads may share a word
-          atomicAdd(&s_stats[0], 1ull);
-          const unsigned long long nk = gain_key(g, t);
-          if (nk > floor_key) {  // a new best exact key: tell the cluster
-            const unsigned long long tagged = tag_key(nk, step);
-            for (int r = 0; r < a.C; ++r)
-              red_dsmem_max_u64(map_rank(smem_addr(&s_hint), r), tagged);
+          if (lane == 0) {
+            ub[tl] = g;
+            atomicOr(&fresh[tl >> 5], 1u << (tl & 31));  // quads may share a word
+            atomicAdd(&s_stats[0], 1ull);
           }
+          const unsigned long long nk = gain_key(g, t);
+          if (nk > floor_key && lane < a.C)  // a new best exact key: lane r tells block r
+            red_dsmem_max_u64(map_rank(smem_addr(&s_hint), (uint32_t)lane), tag_key(nk, step));
         }
         quad_sync(k);
         if (w == 4 * k + ((tl >> 8) & 3)) warp_rescan();  // the warp holding t
@@ -835,7 +836,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
         atomicMax(&s_G[slot], s_qkey[k]);
         if (s_qfresh[k]) atomicMax(&s_BF[slot], s_qkey[k]);
       }
-      if (threadIdx.x == 0) s_H = untag_key(ld_volatile_u64(&s_hint), step);
+      if (threadIdx.x == 0) s_H[slot] = untag_key(ld_volatile_u64(&s_hint), step);
       __syncthreads();
     }
 
