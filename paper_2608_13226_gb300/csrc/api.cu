@@ -267,7 +267,7 @@ static int run_front(const void* feats, int dtype, const float* pos, const int32
     CP_TRY(launch_scene_stats(pos, frame, B, N, stats, s));
     CP_TRY(launch_inv_norms(feats, dtype, pos, B, N, D, at<float>(ws, pl.inv),
                             at<float4>(ws, pl.tok), s));
-    CP_TRY(launch_knn(pos, B, N, d.kk, at<int32_t>(ws, pl.nbr), stats, s));
+    CP_TRY(launch_knn(pos, at<float4>(ws, pl.tok), B, N, d.kk, at<int32_t>(ws, pl.nbr), stats, s));
   }
   {
     Stage st(CP_STAGE_GRAM, s);
@@ -524,7 +524,7 @@ int coverprune_knn(const float* pos, int64_t B, int64_t N, int64_t k, int32_t* n
   SceneStats* stats = at<SceneStats>(ws, align_up(256));
   CP_TRY(cuda_status(cudaMemsetAsync(ws, 0, sizeof(int), s)));
   CP_TRY(launch_scene_stats(pos, nullptr, B, N, stats, s));  // frames are not needed
-  CP_TRY(launch_knn(pos, B, N, (int)k, k > 0 ? nbr : nullptr, stats, s));
+  CP_TRY(launch_knn(pos, nullptr, B, N, (int)k, k > 0 ? nbr : nullptr, stats, s));
   if (diameter) CP_TRY(launch_diameter(stats, B, diameter, s));
   return CP_OK;
 }

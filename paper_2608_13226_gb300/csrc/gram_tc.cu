@@ -15,9 +15,12 @@
 //               one of two 128x256 fp32 accumulators (double buffer)
 //   warps 2..9  epilogue: warps w and w+4 share TMEM lane quadrant w%4 and
 //               split the 256 columns; tcgen05.ld 32 lanes x 32 columns at a
-//               time, FST arithmetic in registers, 16-byte stores (or the
-//               min/max); the 32 columns' token data is staged per warp in
-//               shared memory
+//               time, FST arithmetic in registers (or the min/max); the 32
+//               columns' token data is staged per warp in shared memory.
+//               Cost rows leave through a per-warp 32 x 16 shared-memory
+//               transpose, so that each store instruction writes 8 rows x
+//               64 contiguous bytes: whole sectors, which L2 takes without
+//               first reading the rest of a sector from DRAM
 // Stage hand-offs use mbarriers; the accumulator hand-off uses
 // tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
 // time limit: on expiry the kernel records CP_ETIMEOUT, stops issuing work,
@@ -37,7 +40,10 @@ constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
 constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;  // 32 KB
 constexpr uint32_t TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
 constexpr uint32_t TC_TMEM_COLS = 512;              // 2 accumulators x 256 fp32 columns
-constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES + 1024;  // + alignment slack
+constexpr uint32_t TC_STG_FLOATS = 32 * 16;         // epilogue staging per warp (2 KB)
+constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES +
+                           (size_t)TC_EPI_WARPS * TC_STG_FLOATS * sizeof(float) +
+                           1024;  // + alignment slack
 
 enum { TC_MINMAX = 0, TC_COST = 1 };
 
@@ -56,6 +62,7 @@ struct TcArgs {
   DevParams P;
   float* cost;
   int64_t ldc;
+  int vec_ok;             // cost rows take 16-byte stores (ldc % 4 == 0, 16-byte base)
   SceneStats* stats;
   int* status;
   int N, B, TI, TJ, num_kb, tiles_per_scene, total_tiles;
@@ -345,6 +352,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const int half = (warp - 2) / 4;               // which 128 of the 256 columns
     const int ew = warp - 2;                       // epilogue warp index (staging slot)
     const int r = q * 32 + lane;                   // row of the tile
+    float* stg = reinterpret_cast<float*>(smem_raw + (smem_base - smem_u32(smem_raw)) +
+                                          TC_STAGES * TC_STAGE_BYTES) +
+                 ew * TC_STG_FLOATS;               // this warp's 32 x 16 staging tile
     const float log2_scale = 0.69314718055994531f * a.P.inv_log1p_kappa;
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -376,11 +386,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (MODE == TC_COST) taui = __ldg(a.frame + sb + gi);
       }
       SceneNorms nm;
-      float* crow = nullptr;
-      if (MODE == TC_COST) {
-        nm = a.norms[b];
-        crow = a.cost + (sb + (size_t)(row_ok ? gi : 0)) * (size_t)a.ldc;
-      }
+      if (MODE == TC_COST) nm = a.norms[b];
       const uint32_t row_taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN);
 #pragma unroll 1
       for (int c = half * 4; c < half * 4 + 4; ++c) {
@@ -428,16 +434,43 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               }
               v[e] = __float_as_uint(out);
             }
-            if ((a.ldc & 3) == 0 && j0 + 32 <= a.ldc) {
-              float4* dst = reinterpret_cast<float4*>(crow + j0);
+          }
+        }
+        if (MODE == TC_COST) {
+          // two 16-column halves through the staging tile: lane l writes row
+          // l's four float4 chunks (chunk c at c ^ ((l >> 1) & 3), so a phase
+          // of 8 lanes hits 8 distinct bank groups), then store i (of 4)
+          // moves rows 8i + l/4, chunk l % 4: 8 rows x 64 bytes
+          const int r0 = I * TC_BM + q * 32;  // first row of this warp
 #pragma unroll
-              for (int e = 0; e < 8; ++e)
-                dst[e] = make_float4(__uint_as_float(v[4 * e]), __uint_as_float(v[4 * e + 1]),
-                                     __uint_as_float(v[4 * e + 2]), __uint_as_float(v[4 * e + 3]));
-            } else {
+          for (int h = 0; h < 2; ++h) {
+            __syncwarp();  // the previous half's loads are done
 #pragma unroll
-              for (int e = 0; e < 32; ++e)
-                if (j0 + e < a.ldc) crow[j0 + e] = __uint_as_float(v[e]);
+            for (int c = 0; c < 4; ++c) {
+              const int e = 16 * h + 4 * c;
+              *reinterpret_cast<float4*>(stg + lane * 16 + 4 * (c ^ ((lane >> 1) & 3))) =
+                  make_float4(__uint_as_float(v[e]), __uint_as_float(v[e + 1]),
+                              __uint_as_float(v[e + 2]), __uint_as_float(v[e + 3]));
+            }
+            __syncwarp();  // this half's rows are all written
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int rr = 8 * i + (lane >> 2), c = lane & 3;  // rr < 32
+              const float4 val =
+                  *reinterpret_cast<const float4*>(stg + rr * 16 + 4 * (c ^ ((rr >> 1) & 3)));
+              const int grow = r0 + rr;
+              const int col = j0 + 16 * h + 4 * c;
+              if (grow < a.N && col < a.ldc) {
+                float* dst = a.cost + (sb + (size_t)grow) * (size_t)a.ldc + col;
+                if (a.vec_ok) {  // col % 4 == 0 and ldc % 4 == 0: the chunk fits
+                  *reinterpret_cast<float4*>(dst) = val;
+                } else {
+                  dst[0] = val.x;
+                  if (col + 1 < a.ldc) dst[1] = val.y;
+                  if (col + 2 < a.ldc) dst[2] = val.z;
+                  if (col + 3 < a.ldc) dst[3] = val.w;
+                }
+              }
             }
           }
         }
@@ -533,6 +566,7 @@ int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const 
   a.P = P;
   a.cost = cost;
   a.ldc = ldc;
+  a.vec_ok = (ldc % 4 == 0) && (reinterpret_cast<uintptr_t>(cost) % 16 == 0);
   a.stats = stats;
   a.status = status;
   a.N = (int)N;

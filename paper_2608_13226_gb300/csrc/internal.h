@@ -78,7 +78,7 @@ int launch_inv_norms(const void* feats, int dtype, const float* pos, int64_t B, 
                      int64_t D, float* inv, float4* tok, cudaStream_t s);
 // K1: per token the kk nearest other tokens by (fp32 d^2, index) into
 // nbr[(b*N + j)*kk + q]; also the scene's largest squared distance.
-int launch_knn(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
+int launch_knn(const float* pos, const float4* tok, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
                cudaStream_t s);
 // K2 (fp32 SIMT and bf16 tensor-core variants): max and min cosine over all
 // pairs into stats.

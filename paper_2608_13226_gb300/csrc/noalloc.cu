@@ -83,7 +83,7 @@ extern "C" int coverprune_knn_noalloc(const float* pos, int64_t B, int64_t N, in
   CP_TRY_STATUS(cuda_status(cudaMemsetAsync(base, 0, sizeof(int), s),
                             "coverprune_knn_noalloc: status"));
   CP_TRY_STATUS(launch_scene_stats(pos, nullptr, B, N, stats, s));
-  CP_TRY_STATUS(launch_knn(pos, B, N, (int)k, k > 0 ? nbr : nullptr, stats, s));
+  CP_TRY_STATUS(launch_knn(pos, nullptr, B, N, (int)k, k > 0 ? nbr : nullptr, stats, s));
   if (diameter) CP_TRY_STATUS(launch_diameter(stats, B, diameter, s));
   return CP_OK;
 }

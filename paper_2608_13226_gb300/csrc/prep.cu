@@ -279,13 +279,119 @@ __global__ void __launch_bounds__(256) k_knn_warp(const float* __restrict__ pos,
   }
 }
 
-int launch_knn(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
-               cudaStream_t s) {
+// K1 for kk <= 8, two tokens per warp: each candidate position is loaded
+// once (as a float4 from the token table when one is given) for both query
+// rows; the quick test on the d^2 bits skips the 64-bit key compare for
+// almost every candidate.  Same keys, same lists as k_knn_warp.
+template <int KK, bool TOK>
+__global__ void __launch_bounds__(256) k_knn_pair(const float* __restrict__ pos,
+                                                  const float4* __restrict__ tok, int N, int kk,
+                                                  int32_t* __restrict__ nbr, SceneStats* stats) {
+  const int j0 = (blockIdx.x * 8 + (threadIdx.x >> 5)) * 2;
+  const int b = blockIdx.y;
+  const int lane = threadIdx.x & 31;
+  const float* X = pos + (size_t)b * N * 3;
+  const float4* T = TOK ? tok + (size_t)b * N : nullptr;
+  uint32_t dmax = 0u;
+  if (j0 < N) {
+    const bool two = j0 + 1 < N;
+    const int j1 = two ? j0 + 1 : j0;
+    const float ax = X[3 * j0], ay = X[3 * j0 + 1], az = X[3 * j0 + 2];
+    const float bx = X[3 * j1], by = X[3 * j1 + 1], bz = X[3 * j1 + 2];
+    unsigned long long best0[KK], best1[KK];
+#pragma unroll
+    for (int i = 0; i < KK; ++i) best0[i] = best1[i] = ~0ull;
+    for (int k = lane; k < N; k += 32) {
+      float px, py, pz;
+      if (TOK) {
+        const float4 p = __ldg(T + k);
+        px = p.x;
+        py = p.y;
+        pz = p.z;
+      } else {
+        px = __ldg(X + 3 * k);
+        py = __ldg(X + 3 * k + 1);
+        pz = __ldg(X + 3 * k + 2);
+      }
+      const uint32_t ba = __float_as_uint(sqdist_rn(ax, ay, az, px, py, pz));
+      const uint32_t bb = __float_as_uint(sqdist_rn(bx, by, bz, px, py, pz));
+      dmax = max(dmax, max(ba, bb));
+      if (ba <= (uint32_t)(best0[KK - 1] >> 32) && k != j0) {
+        const unsigned long long key = ((unsigned long long)ba << 32) | (uint32_t)k;
+        if (key < best0[KK - 1]) {
+          best0[KK - 1] = key;
+#pragma unroll
+          for (int i = KK - 1; i > 0; --i)
+            if (best0[i] < best0[i - 1]) {
+              const unsigned long long t = best0[i];
+              best0[i] = best0[i - 1];
+              best0[i - 1] = t;
+            }
+        }
+      }
+      if (bb <= (uint32_t)(best1[KK - 1] >> 32) && k != j1) {
+        const unsigned long long key = ((unsigned long long)bb << 32) | (uint32_t)k;
+        if (key < best1[KK - 1]) {
+          best1[KK - 1] = key;
+#pragma unroll
+          for (int i = KK - 1; i > 0; --i)
+            if (best1[i] < best1[i - 1]) {
+              const unsigned long long t = best1[i];
+              best1[i] = best1[i - 1];
+              best1[i - 1] = t;
+            }
+        }
+      }
+    }
+    if (nbr) {
+      int32_t* out0 = nbr + ((size_t)b * N + j0) * kk;
+      for (int q = 0; q < kk; ++q) {
+        const unsigned long long m = warp_min_u64(best0[0]);
+        if (lane == 0) out0[q] = (int32_t)(m & 0xFFFFFFFFull);
+        if (best0[0] == m) {  // keys are unique: exactly one lane pops its head
+#pragma unroll
+          for (int i = 0; i < KK - 1; ++i) best0[i] = best0[i + 1];
+          best0[KK - 1] = ~0ull;
+        }
+      }
+      if (two) {
+        int32_t* out1 = nbr + ((size_t)b * N + j1) * kk;
+        for (int q = 0; q < kk; ++q) {
+          const unsigned long long m = warp_min_u64(best1[0]);
+          if (lane == 0) out1[q] = (int32_t)(m & 0xFFFFFFFFull);
+          if (best1[0] == m) {
+#pragma unroll
+            for (int i = 0; i < KK - 1; ++i) best1[i] = best1[i + 1];
+            best1[KK - 1] = ~0ull;
+          }
+        }
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) dmax = max(dmax, __shfl_xor_sync(0xFFFFFFFFu, dmax, o));
+  __shared__ uint32_t s_dmax[8];
+  if (lane == 0) s_dmax[threadIdx.x >> 5] = dmax;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t m = s_dmax[0];
+    for (int i = 1; i < 8; ++i) m = max(m, s_dmax[i]);
+    atomicMax(&stats[b].d2_max_bits, m);
+  }
+}
+
+int launch_knn(const float* pos, const float4* tok, int64_t B, int64_t N, int kk, int32_t* nbr,
+               SceneStats* stats, cudaStream_t s) {
+  if (kk <= 8) {
+    dim3 grid((unsigned)((N + 15) / 16), (unsigned)B);
+    if (tok)
+      k_knn_pair<8, true><<<grid, 256, 0, s>>>(pos, tok, (int)N, kk, nbr, stats);
+    else
+      k_knn_pair<8, false><<<grid, 256, 0, s>>>(pos, nullptr, (int)N, kk, nbr, stats);
+    return last_launch_status();
+  }
   if (kk <= 32) {
     dim3 grid((unsigned)((N + 7) / 8), (unsigned)B);
-    if (kk <= 8)
-      k_knn_warp<8><<<grid, 256, 0, s>>>(pos, (int)N, kk, nbr, stats);
-    else if (kk <= 16)
+    if (kk <= 16)
       k_knn_warp<16><<<grid, 256, 0, s>>>(pos, (int)N, kk, nbr, stats);
     else
       k_knn_warp<32><<<grid, 256, 0, s>>>(pos, (int)N, kk, nbr, stats);

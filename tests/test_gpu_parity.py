@@ -91,6 +91,24 @@ def test_cost_bf16_ragged(orc, N, D, seed):
     assert_capacity_close(host(out["capacity"]), vo, "bf16")
 
 
+def test_cost_output_offset_by_one_float():
+    """An output whose base is 4-byte but not 16-byte aligned (a slice one
+    float into a buffer) gets the same cost as an aligned one: the kernel
+    falls back from 16-byte stores when the base or the row stride forbids
+    them."""
+    s = scene("short_clip", 9, N=256, D=128)
+    f, pos, fr = to_dev(s)
+    ref = cp.coverprune_cost(f, pos, fr, cp.Params(), capacity=False, norms=False)["cost"]
+    buf = torch.full((256 * 256 + 1,), -1.0, dtype=torch.float32, device="cuda")
+    shifted = buf[1:].view(256, 256)
+    assert shifted.data_ptr() % 16 == 4
+    cp.coverprune_cost(f, pos, fr, cp.Params(), capacity=False, norms=False,
+                       out={"cost": shifted})
+    torch.cuda.synchronize()
+    assert torch.equal(shifted, ref)
+    assert buf[0].item() == -1.0
+
+
 def test_cost_ablation_weights(orc):
     s = scene("short_clip", 3, N=500, D=256)
     prm = cp.Params(lambda_f=0.5, lambda_x=2.0, lambda_tau=0.0, kappa=3.0, alpha_f=0.2,
