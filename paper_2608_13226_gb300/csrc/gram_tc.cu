@@ -17,10 +17,10 @@
 //               split the 256 columns; tcgen05.ld 32 lanes x 32 columns at a
 //               time, FST arithmetic in registers (or the min/max); the 32
 //               columns' token data is staged per warp in shared memory.
-//               Cost rows leave through a per-warp 32 x 16 shared-memory
-//               transpose, so that each store instruction writes 8 rows x
-//               64 contiguous bytes: whole sectors, which L2 takes without
-//               first reading the rest of a sector from DRAM
+//               Cost rows leave through a per-warp 32 x 32 shared-memory
+//               transpose (the same 4 KB that held the token data), so that
+//               each store instruction writes 4 rows x 128 contiguous bytes:
+//               whole L2 lines, which L2 takes without reading DRAM first
 // Stage hand-offs use mbarriers; the accumulator hand-off uses
 // tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
 // time limit: on expiry the kernel records CP_ETIMEOUT, stops issuing work,
@@ -40,7 +40,7 @@ constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
 constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;  // 32 KB
 constexpr uint32_t TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
 constexpr uint32_t TC_TMEM_COLS = 512;              // 2 accumulators x 256 fp32 columns
-constexpr uint32_t TC_STG_FLOATS = 32 * 16;         // epilogue staging per warp (2 KB)
+constexpr uint32_t TC_STG_FLOATS = 32 * 32;         // epilogue staging per warp (4 KB)
 constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES +
                            (size_t)TC_EPI_WARPS * TC_STG_FLOATS * sizeof(float) +
                            1024;  // + alignment slack
@@ -118,13 +118,32 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
 }
 
 // ---- TMA ---------------------------------------------------------------------
+// L2 policies: the feature operands are re-read by every tile of a scene and
+// should stay in L2 (evict last); each cost line is written once (evict
+// first), so the output stream does not push the features out.
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
 __device__ __forceinline__ void tma_load_3d(const CUtensorMap* map, uint64_t* bar, uint32_t dst,
-                                            int x, int y, int z) {
+                                            int x, int y, int z, uint64_t policy) {
   asm volatile(
       "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)),
+      "l"(policy)
       : "memory");
+}
+__device__ __forceinline__ void st_f4_policy(float* p, const float4& v, uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x),
+               "f"(v.y), "f"(v.z), "f"(v.w), "l"(policy)
+               : "memory");
 }
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -230,8 +249,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2];
   __shared__ uint32_t s_tmem_base;
   __shared__ volatile int s_abort;
-  __shared__ float4 s_col[TC_EPI_WARPS][32];  // per epilogue warp: (x, y, z, 1/||f||)
-  __shared__ int s_tau[TC_EPI_WARPS][32];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t smem_base = (smem_u32(smem_raw) + 1023u) & ~1023u;  // 1024-B aligned ring
@@ -265,6 +282,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
+      const uint64_t keep = l2_policy_evict_last();
       int stage = 0;
       uint32_t phase = 0;
       uint32_t pending = 0;        // stages holding a load not yet seen consumed
@@ -277,8 +295,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           pending &= ~(1u << stage);
           const uint32_t sa = smem_base + (uint32_t)stage * TC_STAGE_BYTES;
           mbar_arrive_expect_tx(&full_bar[stage], TC_STAGE_BYTES);
-          tma_load_3d(&mapA, &full_bar[stage], sa, kb * TC_BK, I * TC_BM, b);
-          tma_load_3d(&mapB, &full_bar[stage], sa + TC_A_BYTES, kb * TC_BK, J * TC_BN, b);
+          tma_load_3d(&mapA, &full_bar[stage], sa, kb * TC_BK, I * TC_BM, b, keep);
+          tma_load_3d(&mapB, &full_bar[stage], sa + TC_A_BYTES, kb * TC_BK, J * TC_BN, b, keep);
           pending |= 1u << stage;
           pend_parity = (pend_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == TC_STAGES) {
@@ -354,8 +372,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const int r = q * 32 + lane;                   // row of the tile
     float* stg = reinterpret_cast<float*>(smem_raw + (smem_base - smem_u32(smem_raw)) +
                                           TC_STAGES * TC_STAGE_BYTES) +
-                 ew * TC_STG_FLOATS;               // this warp's 32 x 16 staging tile
+                 ew * TC_STG_FLOATS;               // this warp's 32 x 32 staging tile
+    float4* s_col = reinterpret_cast<float4*>(stg);  // chunk columns: (x, y, z, 1/||f||)
+    int* s_tau = reinterpret_cast<int*>(stg + 4 * 32);  // ... and their frames
     const float log2_scale = 0.69314718055994531f * a.P.inv_log1p_kappa;
+    const uint64_t stream_out = l2_policy_evict_first();
     int acc = 0;
     uint32_t acc_phase = 0;
     float cmax = -INFINITY, cmin = INFINITY;
@@ -400,9 +421,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             tj = __ldg(a.tok + sb + jl);
             if (MODE == TC_COST) tauj = __ldg(a.frame + sb + jl);
           }
-          __syncwarp();
-          s_col[ew][lane] = tj;
-          s_tau[ew][lane] = tauj;
+          __syncwarp();  // the previous chunk's staging reads are done
+          s_col[lane] = tj;
+          s_tau[lane] = tauj;
           __syncwarp();
         }
         uint32_t v[32];
@@ -413,7 +434,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             for (int e = 0; e < 32; ++e) {
               const int j = j0 + e;
               if (j < a.N) {
-                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * s_col[ew][e].w);
+                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * s_col[e].w);
                 if (j == gi && ti.w > 0.0f) cv = 1.0f;  // cos(f, f) = 1 exactly
                 cmax = fmaxf(cmax, cv);
                 cmin = fminf(cmin, cv);
@@ -425,51 +446,44 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               const int j = j0 + e;
               float out = 0.0f;  // pad columns N <= j < ldc hold 0
               if (j < a.N) {
-                const float4 tj = s_col[ew][e];
+                const float4 tj = s_col[e];
                 float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * tj.w);
                 if (j == gi && ti.w > 0.0f) cv = 1.0f;
                 const float dx = ti.x - tj.x, dy = ti.y - tj.y, dz = ti.z - tj.z;
                 const float d2 = dx * dx + dy * dy + dz * dz;
-                out = fst_cost_fast(cv, d2, taui, s_tau[ew][e], nm, a.P, log2_scale);
+                out = fst_cost_fast(cv, d2, taui, s_tau[e], nm, a.P, log2_scale);
               }
               v[e] = __float_as_uint(out);
             }
           }
         }
         if (MODE == TC_COST) {
-          // two 16-column halves through the staging tile: lane l writes row
-          // l's four float4 chunks (chunk c at c ^ ((l >> 1) & 3), so a phase
-          // of 8 lanes hits 8 distinct bank groups), then store i (of 4)
-          // moves rows 8i + l/4, chunk l % 4: 8 rows x 64 bytes
+          // lane l writes row l's eight float4 chunks (chunk c at c ^ (l & 7),
+          // so a phase of 8 lanes hits 8 distinct bank groups); store i (of
+          // 8) then moves rows 4i + l/8, chunk l % 8: 4 rows x 128 bytes
           const int r0 = I * TC_BM + q * 32;  // first row of this warp
+          __syncwarp();  // every lane is done with the token data
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            __syncwarp();  // the previous half's loads are done
+          for (int c = 0; c < 8; ++c)
+            *reinterpret_cast<float4*>(stg + lane * 32 + 4 * (c ^ (lane & 7))) =
+                make_float4(__uint_as_float(v[4 * c]), __uint_as_float(v[4 * c + 1]),
+                            __uint_as_float(v[4 * c + 2]), __uint_as_float(v[4 * c + 3]));
+          __syncwarp();
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-              const int e = 16 * h + 4 * c;
-              *reinterpret_cast<float4*>(stg + lane * 16 + 4 * (c ^ ((lane >> 1) & 3))) =
-                  make_float4(__uint_as_float(v[e]), __uint_as_float(v[e + 1]),
-                              __uint_as_float(v[e + 2]), __uint_as_float(v[e + 3]));
-            }
-            __syncwarp();  // this half's rows are all written
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int rr = 8 * i + (lane >> 2), c = lane & 3;  // rr < 32
-              const float4 val =
-                  *reinterpret_cast<const float4*>(stg + rr * 16 + 4 * (c ^ ((rr >> 1) & 3)));
-              const int grow = r0 + rr;
-              const int col = j0 + 16 * h + 4 * c;
-              if (grow < a.N && col < a.ldc) {
-                float* dst = a.cost + (sb + (size_t)grow) * (size_t)a.ldc + col;
-                if (a.vec_ok) {  // col % 4 == 0 and ldc % 4 == 0: the chunk fits
-                  *reinterpret_cast<float4*>(dst) = val;
-                } else {
-                  dst[0] = val.x;
-                  if (col + 1 < a.ldc) dst[1] = val.y;
-                  if (col + 2 < a.ldc) dst[2] = val.z;
-                  if (col + 3 < a.ldc) dst[3] = val.w;
-                }
+          for (int i = 0; i < 8; ++i) {
+            const int rr = 4 * i + (lane >> 3), c = lane & 7;  // rr < 32
+            const float4 val = *reinterpret_cast<const float4*>(stg + rr * 32 + 4 * (c ^ (rr & 7)));
+            const int grow = r0 + rr;
+            const int col = j0 + 4 * c;
+            if (grow < a.N && col < a.ldc) {
+              float* dst = a.cost + (sb + (size_t)grow) * (size_t)a.ldc + col;
+              if (a.vec_ok) {  // col % 4 == 0 and ldc % 4 == 0: the chunk fits
+                st_f4_policy(dst, val, stream_out);
+              } else {
+                dst[0] = val.x;
+                if (col + 1 < a.ldc) dst[1] = val.y;
+                if (col + 2 < a.ldc) dst[2] = val.z;
+                if (col + 3 < a.ldc) dst[3] = val.w;
               }
             }
           }
