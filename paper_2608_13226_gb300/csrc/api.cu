@@ -188,6 +188,7 @@ static DevParams dev_params(const cp_params* p, int64_t N) {
 // ---------------------------------------------------------------------------
 struct Plan {
   size_t hdr, counters, stats, norms, inv, tok, nbr, r, v;
+  size_t grid_info, grid_start, grid_pts;         // neighbour grid (kk <= 8)
   size_t cost, slab, partials, order32;           // select
   size_t perm, prefix, gs, proto, score;          // lite
   size_t total;
@@ -195,6 +196,14 @@ struct Plan {
 };
 
 static size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Workspace of coverprune_knn: status block, scene statistics, the grid.
+static size_t knn_ws_bytes(int64_t B, int64_t N) {
+  return align_up(256) + align_up(sizeof(SceneStats) * (size_t)B) +
+         align_up(sizeof(GridInfo) * (size_t)B) +
+         align_up(sizeof(int32_t) * (size_t)B * (size_t)(grid_cells_max(N) + 1)) +
+         align_up(sizeof(float4) * (size_t)B * (size_t)N);
+}
 
 static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d, Plan* pl) {
   memset(pl, 0, sizeof(*pl));
@@ -213,6 +222,11 @@ static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d,
   pl->inv = take(sizeof(float) * BN);
   pl->tok = take(sizeof(float4) * BN);
   pl->nbr = take(sizeof(int32_t) * BN * (size_t)d.kk);
+  if (d.kk <= 8) {
+    pl->grid_info = take(sizeof(GridInfo) * (size_t)B);
+    pl->grid_start = take(sizeof(int32_t) * (size_t)B * (size_t)(grid_cells_max(N) + 1));
+    pl->grid_pts = take(sizeof(float4) * BN);
+  }
   pl->r = take(sizeof(float) * BN);
   pl->v = take(sizeof(float) * BN);
   if (op == CP_OP_SELECT) {
@@ -267,7 +281,13 @@ static int run_front(const void* feats, int dtype, const float* pos, const int32
     CP_TRY(launch_scene_stats(pos, frame, B, N, stats, s));
     CP_TRY(launch_inv_norms(feats, dtype, pos, B, N, D, at<float>(ws, pl.inv),
                             at<float4>(ws, pl.tok), s));
-    CP_TRY(launch_knn(pos, at<float4>(ws, pl.tok), B, N, d.kk, at<int32_t>(ws, pl.nbr), stats, s));
+    if (d.kk <= 8)
+      CP_TRY(launch_knn_grid(pos, B, N, d.kk, at<int32_t>(ws, pl.nbr), stats,
+                             at<GridInfo>(ws, pl.grid_info), at<int32_t>(ws, pl.grid_start),
+                             at<float4>(ws, pl.grid_pts), s));
+    else
+      CP_TRY(launch_knn(pos, at<float4>(ws, pl.tok), B, N, d.kk, at<int32_t>(ws, pl.nbr), stats,
+                        s));
   }
   {
     Stage st(CP_STAGE_GRAM, s);
@@ -347,7 +367,7 @@ int coverprune_workspace_size(int op, int64_t B, int64_t N, int64_t D, int64_t K
     return CP_EINVAL;
   if (op == CP_OP_KNN) {
     if (B < 0 || N < 0 || B > 65535 || N > kMaxKnnN) return CP_EINVAL;
-    *bytes = align_up(256) + align_up(sizeof(SceneStats) * (size_t)(B > 0 ? B : 1));
+    *bytes = knn_ws_bytes(B > 0 ? B : 1, N);
     return CP_OK;
   }
   CP_TRY(check_shapes(dtype, B, N, D, op == CP_OP_COST ? 0 : K));
@@ -518,13 +538,21 @@ int coverprune_knn(const float* pos, int64_t B, int64_t N, int64_t k, int32_t* n
   int64_t L = 2;
   while (L < k) L <<= 1;
   if (8 * L + 4 * N > 200 * 1024) return CP_EUNSUPPORTED;
-  const size_t need = align_up(256) + align_up(sizeof(SceneStats) * (size_t)B);
-  if (!ws || !aligned(ws, 256) || ws_bytes < need) return CP_EWORKSPACE;
+  if (!ws || !aligned(ws, 256) || ws_bytes < knn_ws_bytes(B, N)) return CP_EWORKSPACE;
   cudaStream_t s = (cudaStream_t)stream;
-  SceneStats* stats = at<SceneStats>(ws, align_up(256));
+  const size_t st_off = align_up(256);
+  const size_t gi_off = st_off + align_up(sizeof(SceneStats) * (size_t)B);
+  const size_t gs_off = gi_off + align_up(sizeof(GridInfo) * (size_t)B);
+  const size_t gp_off = gs_off + align_up(sizeof(int32_t) * (size_t)B * (grid_cells_max(N) + 1));
+  SceneStats* stats = at<SceneStats>(ws, st_off);
   CP_TRY(cuda_status(cudaMemsetAsync(ws, 0, sizeof(int), s)));
   CP_TRY(launch_scene_stats(pos, nullptr, B, N, stats, s));  // frames are not needed
-  CP_TRY(launch_knn(pos, nullptr, B, N, (int)k, k > 0 ? nbr : nullptr, stats, s));
+  if (k <= 8)
+    CP_TRY(launch_knn_grid(pos, B, N, (int)k, k > 0 ? nbr : nullptr, stats,
+                           at<GridInfo>(ws, gi_off), at<int32_t>(ws, gs_off),
+                           at<float4>(ws, gp_off), s));
+  else
+    CP_TRY(launch_knn(pos, nullptr, B, N, (int)k, nbr, stats, s));
   if (diameter) CP_TRY(launch_diameter(stats, B, diameter, s));
   return CP_OK;
 }

@@ -45,6 +45,27 @@ struct SceneStats {
 };
 static_assert(sizeof(SceneStats) == 64, "SceneStats layout");
 
+// Uniform grid of one scene for the neighbour search (32 bytes).
+struct GridInfo {
+  float lo[3];   // bounding-box minimum
+  float h;       // cell side
+  float inv_h;
+  int dims[3];   // cells per axis
+  int ncells;
+  int pad;
+};
+static_assert(sizeof(GridInfo) == 40, "GridInfo layout");
+
+// Cell coordinate of x along axis a, clamped to the grid.
+__host__ __device__ inline int grid_coord(const GridInfo& g, float x, int a) {
+  const int c = (int)floorf((x - g.lo[a]) * g.inv_h);
+  return c < 0 ? 0 : (c >= g.dims[a] ? g.dims[a] - 1 : c);
+}
+__host__ __device__ inline int grid_cell(const GridInfo& g, const float* p) {
+  return (grid_coord(g, p[2], 2) * g.dims[1] + grid_coord(g, p[1], 1)) * g.dims[0] +
+         grid_coord(g, p[0], 0);
+}
+
 constexpr double kRangeEps = 1e-6;
 
 // Layout of the 256-byte status block at the start of every workspace
@@ -78,6 +99,10 @@ int launch_inv_norms(const void* feats, int dtype, const float* pos, int64_t B, 
                      int64_t D, float* inv, float4* tok, cudaStream_t s);
 // K1: per token the kk nearest other tokens by (fp32 d^2, index) into
 // nbr[(b*N + j)*kk + q]; also the scene's largest squared distance.
+int grid_cells_max(int64_t N);
+int launch_knn_grid(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr,
+                    SceneStats* stats, GridInfo* info, int32_t* cell_start, float4* sorted,
+                    cudaStream_t s);
 int launch_knn(const float* pos, const float4* tok, int64_t B, int64_t N, int kk, int32_t* nbr, SceneStats* stats,
                cudaStream_t s);
 // K2 (fp32 SIMT and bf16 tensor-core variants): max and min cosine over all

@@ -279,53 +279,65 @@ __global__ void __launch_bounds__(256) k_knn_warp(const float* __restrict__ pos,
   }
 }
 
-// K1 for kk <= 8, two tokens per warp: each candidate position is loaded
-// once (as a float4 from the token table when one is given) for both query
-// rows; the quick test on the d^2 bits skips the 64-bit key compare for
-// almost every candidate.  Same keys, same lists as k_knn_warp.
+// K1 for kk <= 8, two tokens per warp, 16 per block: the block stages the
+// candidate positions in shared-memory tiles of 2048 (from the float4 token
+// table when one is given, else from the xyz array), so each position is
+// read from L2 once per 16 query rows; the quick test on the d^2 bits skips
+// the 64-bit key compare for almost every candidate.  Same keys, same lists
+// as k_knn_warp.
+constexpr int KNN_TILE = 2048;
+
 template <int KK, bool TOK>
 __global__ void __launch_bounds__(256) k_knn_pair(const float* __restrict__ pos,
                                                   const float4* __restrict__ tok, int N, int kk,
                                                   int32_t* __restrict__ nbr, SceneStats* stats) {
+  __shared__ float4 s_p[KNN_TILE];
   const int j0 = (blockIdx.x * 8 + (threadIdx.x >> 5)) * 2;
   const int b = blockIdx.y;
   const int lane = threadIdx.x & 31;
   const float* X = pos + (size_t)b * N * 3;
   const float4* T = TOK ? tok + (size_t)b * N : nullptr;
+  const bool active = j0 < N;
+  const bool two = j0 + 1 < N;
+  const int j1 = two ? j0 + 1 : j0;
+  float ax = 0.f, ay = 0.f, az = 0.f, bx = 0.f, by = 0.f, bz = 0.f;
+  if (active) {
+    ax = X[3 * j0]; ay = X[3 * j0 + 1]; az = X[3 * j0 + 2];
+    bx = X[3 * j1]; by = X[3 * j1 + 1]; bz = X[3 * j1 + 2];
+  }
   uint32_t dmax = 0u;
-  if (j0 < N) {
-    const bool two = j0 + 1 < N;
-    const int j1 = two ? j0 + 1 : j0;
-    const float ax = X[3 * j0], ay = X[3 * j0 + 1], az = X[3 * j0 + 2];
-    const float bx = X[3 * j1], by = X[3 * j1 + 1], bz = X[3 * j1 + 2];
-    unsigned long long best0[KK], best1[KK];
+  unsigned long long best0[KK], best1[KK];
 #pragma unroll
-    for (int i = 0; i < KK; ++i) best0[i] = best1[i] = ~0ull;
-    for (int k = lane; k < N; k += 32) {
-      float px, py, pz;
+  for (int i = 0; i < KK; ++i) best0[i] = best1[i] = ~0ull;
+  for (int base = 0; base < N; base += KNN_TILE) {
+    const int n = min(KNN_TILE, N - base);
+    __syncthreads();  // the previous tile is consumed
+    for (int i = threadIdx.x; i < n; i += 256) {
       if (TOK) {
-        const float4 p = __ldg(T + k);
-        px = p.x;
-        py = p.y;
-        pz = p.z;
+        s_p[i] = __ldg(T + base + i);
       } else {
-        px = __ldg(X + 3 * k);
-        py = __ldg(X + 3 * k + 1);
-        pz = __ldg(X + 3 * k + 2);
+        const int k = base + i;
+        s_p[i] = make_float4(__ldg(X + 3 * k), __ldg(X + 3 * k + 1), __ldg(X + 3 * k + 2), 0.f);
       }
-      const uint32_t ba = __float_as_uint(sqdist_rn(ax, ay, az, px, py, pz));
-      const uint32_t bb = __float_as_uint(sqdist_rn(bx, by, bz, px, py, pz));
+    }
+    __syncthreads();
+    if (!active) continue;
+    for (int i = lane; i < n; i += 32) {
+      const int k = base + i;
+      const float4 p = s_p[i];
+      const uint32_t ba = __float_as_uint(sqdist_rn(ax, ay, az, p.x, p.y, p.z));
+      const uint32_t bb = __float_as_uint(sqdist_rn(bx, by, bz, p.x, p.y, p.z));
       dmax = max(dmax, max(ba, bb));
       if (ba <= (uint32_t)(best0[KK - 1] >> 32) && k != j0) {
         const unsigned long long key = ((unsigned long long)ba << 32) | (uint32_t)k;
         if (key < best0[KK - 1]) {
           best0[KK - 1] = key;
 #pragma unroll
-          for (int i = KK - 1; i > 0; --i)
-            if (best0[i] < best0[i - 1]) {
-              const unsigned long long t = best0[i];
-              best0[i] = best0[i - 1];
-              best0[i - 1] = t;
+          for (int t = KK - 1; t > 0; --t)
+            if (best0[t] < best0[t - 1]) {
+              const unsigned long long x = best0[t];
+              best0[t] = best0[t - 1];
+              best0[t - 1] = x;
             }
         }
       }
@@ -334,36 +346,36 @@ __global__ void __launch_bounds__(256) k_knn_pair(const float* __restrict__ pos,
         if (key < best1[KK - 1]) {
           best1[KK - 1] = key;
 #pragma unroll
-          for (int i = KK - 1; i > 0; --i)
-            if (best1[i] < best1[i - 1]) {
-              const unsigned long long t = best1[i];
-              best1[i] = best1[i - 1];
-              best1[i - 1] = t;
+          for (int t = KK - 1; t > 0; --t)
+            if (best1[t] < best1[t - 1]) {
+              const unsigned long long x = best1[t];
+              best1[t] = best1[t - 1];
+              best1[t - 1] = x;
             }
         }
       }
     }
-    if (nbr) {
-      int32_t* out0 = nbr + ((size_t)b * N + j0) * kk;
-      for (int q = 0; q < kk; ++q) {
-        const unsigned long long m = warp_min_u64(best0[0]);
-        if (lane == 0) out0[q] = (int32_t)(m & 0xFFFFFFFFull);
-        if (best0[0] == m) {  // keys are unique: exactly one lane pops its head
+  }
+  if (active && nbr) {
+    int32_t* out0 = nbr + ((size_t)b * N + j0) * kk;
+    for (int q = 0; q < kk; ++q) {
+      const unsigned long long m = warp_min_u64(best0[0]);
+      if (lane == 0) out0[q] = (int32_t)(m & 0xFFFFFFFFull);
+      if (best0[0] == m) {  // keys are unique: exactly one lane pops its head
 #pragma unroll
-          for (int i = 0; i < KK - 1; ++i) best0[i] = best0[i + 1];
-          best0[KK - 1] = ~0ull;
-        }
+        for (int i = 0; i < KK - 1; ++i) best0[i] = best0[i + 1];
+        best0[KK - 1] = ~0ull;
       }
-      if (two) {
-        int32_t* out1 = nbr + ((size_t)b * N + j1) * kk;
-        for (int q = 0; q < kk; ++q) {
-          const unsigned long long m = warp_min_u64(best1[0]);
-          if (lane == 0) out1[q] = (int32_t)(m & 0xFFFFFFFFull);
-          if (best1[0] == m) {
+    }
+    if (two) {
+      int32_t* out1 = nbr + ((size_t)b * N + j1) * kk;
+      for (int q = 0; q < kk; ++q) {
+        const unsigned long long m = warp_min_u64(best1[0]);
+        if (lane == 0) out1[q] = (int32_t)(m & 0xFFFFFFFFull);
+        if (best1[0] == m) {
 #pragma unroll
-            for (int i = 0; i < KK - 1; ++i) best1[i] = best1[i + 1];
-            best1[KK - 1] = ~0ull;
-          }
+          for (int i = 0; i < KK - 1; ++i) best1[i] = best1[i + 1];
+          best1[KK - 1] = ~0ull;
         }
       }
     }
@@ -408,6 +420,244 @@ int launch_knn(const float* pos, const float4* tok, int64_t B, int64_t N, int kk
     return CP_ECUDA;
   dim3 grid((unsigned)N, (unsigned)B);
   k_knn<<<grid, KNN_THREADS, smem, s>>>(pos, (int)N, kk, list_len, nbr, stats);
+  return last_launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// K1 through a uniform grid (kk <= 8): exact, with the same keys and lists
+// as the brute-force kernels, but each query visits only the cells around
+// it.  The scene's bounding box is cut into cubic cells of side h =
+// (largest extent) / G with G = the least integer such that 4 G^3 >= N, so
+// at most G^3 cells; points are counting-sorted by cell.  A query scans the
+// shells of cells at Chebyshev distance r = 0, 1, 2, ... from its own cell;
+// every point outside the first r shells is more than r h away along some
+// axis, so once the kk-th best squared distance is below ((r - 1/1024) h)^2
+// (the margin covers the rounding of the cell coordinates) no later point
+// can enter the list.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int grid_side(int N) {
+  int G = 1;
+  while (4 * G * G * G < N) ++G;
+  return G;
+}
+
+// One block per scene: bounding box, cell size, counting sort by cell.
+__global__ void __launch_bounds__(1024) k_grid_build(const float* __restrict__ pos, int N,
+                                                     int gmax, GridInfo* __restrict__ info,
+                                                     int32_t* __restrict__ cell_start,
+                                                     float4* __restrict__ sorted) {
+  extern __shared__ int s_cnt[];  // [gmax + 1]
+  __shared__ float s_red[6][32];
+  const int b = blockIdx.x;
+  const float* X = pos + (size_t)b * N * 3;
+  float lo[3] = {INFINITY, INFINITY, INFINITY}, hi[3] = {-INFINITY, -INFINITY, -INFINITY};
+  for (int j = threadIdx.x; j < N; j += blockDim.x)
+#pragma unroll
+    for (int a = 0; a < 3; ++a) {
+      lo[a] = fminf(lo[a], X[3 * j + a]);
+      hi[a] = fmaxf(hi[a], X[3 * j + a]);
+    }
+  for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+    for (int a = 0; a < 3; ++a) {
+      lo[a] = fminf(lo[a], __shfl_xor_sync(0xFFFFFFFFu, lo[a], o));
+      hi[a] = fmaxf(hi[a], __shfl_xor_sync(0xFFFFFFFFu, hi[a], o));
+    }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  if (l == 0)
+    for (int a = 0; a < 3; ++a) {
+      s_red[a][w] = lo[a];
+      s_red[3 + a][w] = hi[a];
+    }
+  for (int c = threadIdx.x; c <= gmax; c += blockDim.x) s_cnt[c] = 0;
+  __syncthreads();
+  __shared__ GridInfo s_g;
+  if (threadIdx.x == 0) {
+    const int nw = blockDim.x >> 5;
+    for (int i = 1; i < nw; ++i)
+      for (int a = 0; a < 3; ++a) {
+        s_red[a][0] = fminf(s_red[a][0], s_red[a][i]);
+        s_red[3 + a][0] = fmaxf(s_red[3 + a][0], s_red[3 + a][i]);
+      }
+    const int G = grid_side(N);
+    float ext = 0.0f;
+    for (int a = 0; a < 3; ++a) ext = fmaxf(ext, s_red[3 + a][0] - s_red[a][0]);
+    GridInfo g;
+    g.h = ext > 0.0f ? ext / (float)G : 1.0f;
+    g.inv_h = 1.0f / g.h;
+    int nc = 1;
+    for (int a = 0; a < 3; ++a) {
+      g.lo[a] = s_red[a][0];
+      const float e = s_red[3 + a][0] - s_red[a][0];
+      int d = (int)ceilf(e * g.inv_h);
+      d = d < 1 ? 1 : (d > G ? G : d);
+      g.dims[a] = d;
+      nc *= d;
+    }
+    g.ncells = nc;
+    s_g = g;
+    info[b] = g;
+  }
+  __syncthreads();
+  const GridInfo g = s_g;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) atomicAdd(&s_cnt[grid_cell(g, X + 3 * j)], 1);
+  __syncthreads();
+  if (threadIdx.x == 0) {  // exclusive scan; cells <= G^3 <= 13824
+    int run = 0;
+    for (int c = 0; c < g.ncells; ++c) {
+      const int n = s_cnt[c];
+      s_cnt[c] = run;
+      run += n;
+    }
+    s_cnt[g.ncells] = run;
+  }
+  __syncthreads();
+  int32_t* cs = cell_start + (size_t)b * (gmax + 1);
+  for (int c = threadIdx.x; c <= g.ncells; c += blockDim.x) cs[c] = s_cnt[c];
+  __syncthreads();
+  float4* out = sorted + (size_t)b * N;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) {
+    const int slot = atomicAdd(&s_cnt[grid_cell(g, X + 3 * j)], 1);
+    out[slot] = make_float4(X[3 * j], X[3 * j + 1], X[3 * j + 2], __int_as_float(j));
+  }
+}
+
+// One thread per query token.
+template <int KK>
+__global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos, int N, int kk,
+                                                  int gmax, const GridInfo* __restrict__ info,
+                                                  const int32_t* __restrict__ cell_start,
+                                                  const float4* __restrict__ sorted,
+                                                  int32_t* __restrict__ nbr) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  const int b = blockIdx.y;
+  if (j >= N) return;
+  const GridInfo g = info[b];
+  const float* X = pos + (size_t)b * N * 3;
+  const int32_t* cs = cell_start + (size_t)b * (gmax + 1);
+  const float4* P = sorted + (size_t)b * N;
+  const float qx = X[3 * j], qy = X[3 * j + 1], qz = X[3 * j + 2];
+  const int cx = grid_coord(g, qx, 0), cy = grid_coord(g, qy, 1), cz = grid_coord(g, qz, 2);
+  unsigned long long best[KK];
+#pragma unroll
+  for (int i = 0; i < KK; ++i) best[i] = ~0ull;
+  const int rmax = max(g.dims[0], max(g.dims[1], g.dims[2]));
+  for (int r = 0; r <= rmax; ++r) {
+    for (int dz = -r; dz <= r; ++dz) {
+      const int z = cz + dz;
+      if (z < 0 || z >= g.dims[2]) continue;
+      for (int dy = -r; dy <= r; ++dy) {
+        const int y = cy + dy;
+        if (y < 0 || y >= g.dims[1]) continue;
+        const bool face = dz == -r || dz == r || dy == -r || dy == r;
+        for (int dx = -r; dx <= r; dx += (face || r == 0) ? 1 : 2 * r) {
+          const int x = cx + dx;
+          if (x < 0 || x >= g.dims[0]) continue;
+          const int c = (z * g.dims[1] + y) * g.dims[0] + x;
+          for (int s = cs[c], e = cs[c + 1]; s < e; ++s) {
+            const float4 p = P[s];
+            const int k = __float_as_int(p.w);
+            const uint32_t bits = __float_as_uint(sqdist_rn(qx, qy, qz, p.x, p.y, p.z));
+            if (k == j || bits > (uint32_t)(best[KK - 1] >> 32)) continue;
+            const unsigned long long key = ((unsigned long long)bits << 32) | (uint32_t)k;
+            if (key < best[KK - 1]) {
+              best[KK - 1] = key;
+#pragma unroll
+              for (int i = KK - 1; i > 0; --i)
+                if (best[i] < best[i - 1]) {
+                  const unsigned long long t = best[i];
+                  best[i] = best[i - 1];
+                  best[i - 1] = t;
+                }
+            }
+          }
+        }
+      }
+    }
+    unsigned long long kth = ~0ull;  // the kk-th best key so far
+#pragma unroll
+    for (int i = 0; i < KK; ++i)
+      if (i == kk - 1) kth = best[i];
+    if (kth != ~0ull) {
+      const float reach = ((float)r - 1.0f / 1024.0f) * g.h;
+      if (reach > 0.0f && __uint_as_float((uint32_t)(kth >> 32)) < reach * reach) break;
+    }
+  }
+  int32_t* out = nbr + ((size_t)b * N + j) * kk;
+#pragma unroll
+  for (int i = 0; i < KK; ++i)
+    if (i < kk) out[i] = (int32_t)(best[i] & 0xFFFFFFFFull);
+}
+
+// The largest pinned-fp32 squared distance over pairs, into stats.d2_max_bits:
+// block of 256 rows, candidate tiles of 1024 in shared memory, only tiles
+// that reach past the block's first row (d^2 is symmetric).
+__global__ void __launch_bounds__(256) k_diameter_pairs(const float* __restrict__ pos, int N,
+                                                        SceneStats* stats) {
+  __shared__ float4 s_p[1024];
+  __shared__ uint32_t s_m[8];
+  const int b = blockIdx.y;
+  const int row0 = blockIdx.x * 256;
+  const float* X = pos + (size_t)b * N * 3;
+  const int i = row0 + threadIdx.x;
+  float qx = 0.f, qy = 0.f, qz = 0.f;
+  if (i < N) {
+    qx = X[3 * i];
+    qy = X[3 * i + 1];
+    qz = X[3 * i + 2];
+  }
+  uint32_t dmax = 0u;
+  for (int base = (row0 / 1024) * 1024; base < N; base += 1024) {
+    const int n = min(1024, N - base);
+    __syncthreads();
+    for (int t = threadIdx.x; t < n; t += 256) {
+      const int k = base + t;
+      s_p[t] = make_float4(X[3 * k], X[3 * k + 1], X[3 * k + 2], 0.f);
+    }
+    __syncthreads();
+    if (i < N)
+      for (int t = 0; t < n; ++t) {
+        const float4 p = s_p[t];
+        dmax = max(dmax, __float_as_uint(sqdist_rn(qx, qy, qz, p.x, p.y, p.z)));
+      }
+  }
+  for (int o = 16; o > 0; o >>= 1) dmax = max(dmax, __shfl_xor_sync(0xFFFFFFFFu, dmax, o));
+  if ((threadIdx.x & 31) == 0) s_m[threadIdx.x >> 5] = dmax;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t m = s_m[0];
+    for (int w = 1; w < 8; ++w) m = max(m, s_m[w]);
+    atomicMax(&stats[b].d2_max_bits, m);
+  }
+}
+
+int grid_cells_max(int64_t N) {
+  int64_t G = 1;
+  while (4 * G * G * G < N) ++G;
+  return (int)(G * G * G);
+}
+
+int launch_knn_grid(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr,
+                    SceneStats* stats, GridInfo* info, int32_t* cell_start, float4* sorted,
+                    cudaStream_t s) {
+  const int gmax = grid_cells_max(N);
+  {
+    dim3 grid((unsigned)((N + 255) / 256), (unsigned)B);
+    k_diameter_pairs<<<grid, 256, 0, s>>>(pos, (int)N, stats);
+    CP_TRY_STATUS(last_launch_status());
+  }
+  if (kk <= 0) return CP_OK;
+  if (kk > 8) return CP_EINVAL;
+  const size_t smem = sizeof(int) * (size_t)(gmax + 1);
+  if (smem > 48 * 1024 &&
+      cuda_status(cudaFuncSetAttribute(k_grid_build, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem),
+                  "launch_knn_grid: smem attribute") != CP_OK)
+    return CP_ECUDA;
+  k_grid_build<<<(unsigned)B, 1024, smem, s>>>(pos, (int)N, gmax, info, cell_start, sorted);
+  CP_TRY_STATUS(last_launch_status());
+  dim3 grid((unsigned)((N + 127) / 128), (unsigned)B);
+  k_knn_grid<8><<<grid, 128, 0, s>>>(pos, (int)N, kk, gmax, info, cell_start, sorted, nbr);
   return last_launch_status();
 }
 
