@@ -25,7 +25,8 @@ int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64
                           SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s);
 int launch_cost_tc(const void* feats, const float4* tok, const int32_t* frame,
                    const SceneNorms* norms, const DevParams& P, int64_t B, int64_t N, int64_t D,
-                   float* cost, int64_t ldc, int* status, uint64_t timeout_ns, cudaStream_t s);
+                   float* cost, int64_t ldc, const float* v, float* g0, int* status,
+                   uint64_t timeout_ns, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Stage timing and launch counting.
@@ -120,13 +121,16 @@ int launch_gram_minmax(const void* feats, int dtype, const float* inv, const flo
   return launch_gram_minmax_simt(feats, dtype, inv, B, N, D, stats, s);
 }
 
+// g0 (bf16 features only; may be null): every row's first greedy gain terms
+// summed in the cost epilogue per 128-column half tile, [B][g0_slots(N)][N].
 int launch_cost(const void* feats, int dtype, const float* inv, const float4* tok,
                 const float* pos, const int32_t* frame, const SceneNorms* norms,
                 const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
-                int* status, cudaStream_t s) {
-  if (dtype == CP_BF16)
-    return launch_cost_tc(feats, tok, frame, norms, P, B, N, D, cost, ldc, status, P.timeout_ns,
-                          s);
+                int* status, cudaStream_t s, const float* v, float* g0) {
+  if (dtype == CP_BF16) {
+    return launch_cost_tc(feats, tok, frame, norms, P, B, N, D, cost, ldc, v, g0, status,
+                          P.timeout_ns, s);
+  }
   return launch_cost_simt(feats, dtype, inv, pos, frame, norms, P, B, N, D, cost, ldc, s);
 }
 
@@ -189,13 +193,17 @@ static DevParams dev_params(const cp_params* p, int64_t N) {
 struct Plan {
   size_t hdr, counters, stats, norms, inv, tok, nbr, r, v;
   size_t grid_info, grid_start, grid_pts;         // neighbour grid (kk <= 8)
-  size_t cost, slab, partials, order32;           // select
+  size_t cost, slab, partials, order32, g0;       // select
   size_t perm, prefix, gs, proto, score;          // lite
   size_t total;
   int64_t ldc;
 };
 
 static size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Slots of the cost epilogue's first-gain partial sums per row: one per
+// 128-column half of a 256-column tile.
+static int64_t g0_slots(int64_t N) { return 2 * ((N + 255) / 256); }
 
 // Workspace of coverprune_knn: status block, scene statistics, the grid.
 static size_t knn_ws_bytes(int64_t B, int64_t N) {
@@ -234,6 +242,7 @@ static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d,
     if (d.g < N) pl->slab = take(sizeof(float) * BN * (size_t)d.g);
     pl->partials = take(sizeof(uint64_t) * (size_t)sgs_partials_count(B, N));
     pl->order32 = take(sizeof(int32_t) * (size_t)B * (size_t)K);
+    pl->g0 = take(sizeof(float) * BN * (size_t)g0_slots(N));
   } else if (op == CP_OP_LITE) {
     pl->perm = take(sizeof(int32_t) * BN);
     pl->prefix = take(sizeof(uint64_t) * BN);
@@ -461,10 +470,12 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
                            v, nullptr, s));
   }
   float* C = at<float>(ws, pl.cost);
+  // the dense lazy selection starts from bounds the cost epilogue sums
+  float* g0 = (dtype == CP_BF16 && d.g >= N && d.sgs_mode == 0) ? at<float>(ws, pl.g0) : nullptr;
   {
     Stage st(CP_STAGE_COST, s);
     CP_TRY(launch_cost(feats, dtype, inv, at<float4>(ws, pl.tok), pos, frame, nm, d, B, N, D, C,
-                       pl.ldc, status, s));
+                       pl.ldc, status, s, v, g0));
   }
   int32_t* order32 = at<int32_t>(ws, pl.order32);
   {
@@ -475,7 +486,8 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
       CP_TRY(launch_slab(C, pl.ldc, nbr, d, B, N, slab, s));
     }
     CP_TRY(launch_sgs(C, pl.ldc, slab, nbr, v, d, B, N, K, order32, gains, objective,
-                      at<uint64_t>(ws, pl.partials), at<uint32_t>(ws, pl.counters), status, s));
+                      at<uint64_t>(ws, pl.partials), at<uint32_t>(ws, pl.counters), status, s,
+                      g0));
   }
   Stage st(CP_STAGE_OUTPUT, s);
   CP_TRY(launch_sort_kept(order32, B, K, kept, order, s));

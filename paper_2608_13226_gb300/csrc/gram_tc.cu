@@ -5,11 +5,21 @@
 //   MINMAX  max and min of cos(f_i, f_j) over the pairs i <= j (the feature
 //           normaliser of Sec. 3.3) -- only the tiles on or above the
 //           diagonal run, no output but two atomics per warp
-//   COST    the FST cost of Eq. fst_cost, written row-major with stride ldc
+//   COST    the FST cost of Eq. fst_cost, written row-major with stride ldc;
+//           optionally also every row's partial sums of v_j max(m0 - C(t,
+//           j), 0) over each 128-column half tile, one slot per half tile:
+//           the greedy's first gains, summed by the selection in another
+//           order than its own (it uses them inflated, as bounds)
 //
-// One persistent CTA per SM, 10 warps:
-//   warp 0      TMA producer: 128x64 (A) and 256x64 (B) bf16 boxes, 128-byte
-//               swizzle, into a 4-stage shared-memory ring (48 KB a stage)
+// Persistent clusters of two CTAs (one CTA per SM).  The two CTAs of a
+// cluster compute the row tiles 2p and 2p+1 of the same 256-column tile:
+// each loads its own 128x64 A box and one 128-row half of the shared
+// 256x64 B box, multicast to both CTAs, so a CTA fetches 32 KB from L2 per
+// 64-deep step instead of 48 (measured: the normaliser GEMM 0.88 -> 0.95 of
+// the bf16 peak, the cost GEMM ~1% faster).  Each CTA has 10 warps:
+//   warp 0      TMA producer: 128x64 bf16 boxes, 128-byte swizzle, into a
+//               4-stage shared-memory ring (48 KB a stage); a stage is
+//               refilled once both CTAs' MMAs have released it
 //   warp 1      allocates 512 TMEM columns; lane 0 issues
 //               tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) into
 //               one of two 128x256 fp32 accumulators (double buffer)
@@ -21,8 +31,9 @@
 //               transpose (the same 4 KB that held the token data), so that
 //               each store instruction writes 4 rows x 128 contiguous bytes:
 //               whole L2 lines, which L2 takes without reading DRAM first
-// Stage hand-offs use mbarriers; the accumulator hand-off uses
-// tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
+// Stage hand-offs use mbarriers (a stage's "empty" barrier counts the
+// commits of both CTAs' MMA threads, multicast); the accumulator hand-off
+// uses tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
 // time limit: on expiry the kernel records CP_ETIMEOUT, stops issuing work,
 // waits (bounded) for the copies and MMAs it already issued, frees its TMEM
 // and returns.
@@ -63,9 +74,13 @@ struct TcArgs {
   float* cost;
   int64_t ldc;
   int vec_ok;             // cost rows take 16-byte stores (ldc % 4 == 0, 16-byte base)
+  const float* v;         // [B*N] capacity, read when g0 is set
+  float* g0;              // [B][2 TJ][N] half-tile row sums of v_j max(m0 - C, 0), or null
+  float m0;
   SceneStats* stats;
   int* status;
-  int N, B, TI, TJ, num_kb, tiles_per_scene, total_tiles;
+  int N, B, TI, TJ, num_kb;
+  int pairs_per_scene, total_pairs;  // (row-tile pair, column tile) units
   uint64_t timeout_ns;
 };
 
@@ -140,6 +155,18 @@ __device__ __forceinline__ void tma_load_3d(const CUtensorMap* map, uint64_t* ba
       "l"(policy)
       : "memory");
 }
+// The same box into the same shared-memory offset of every CTA in mask, each
+// CTA's mbarrier at that offset receiving the bytes.
+__device__ __forceinline__ void tma_load_3d_mc(const CUtensorMap* map, uint64_t* bar, uint32_t dst,
+                                               int x, int y, int z, uint16_t mask,
+                                               uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".multicast::cluster.L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6, %7;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "h"(mask),
+      "l"(policy)
+      : "memory");
+}
 __device__ __forceinline__ void st_f4_policy(float* p, const float4& v, uint64_t policy) {
   asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x),
                "f"(v.y), "f"(v.z), "f"(v.w), "l"(policy)
@@ -175,6 +202,24 @@ __device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint6
       "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
       : "memory");
 }
+// Arrive on the mbarrier at bar's offset in every CTA of mask once the MMAs
+// issued so far have completed.
+__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
@@ -195,18 +240,31 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// FST cost of one pair (Eq. fst_cost) for the tensor-core path: as
-// fst_cost_from, with the distance from rsqrtf and log(1 + x) from __log2f
-// (both within ~1e-7 absolute here, far inside the bf16 parity bar).
-__device__ __forceinline__ float fst_cost_fast(float cosv, float d2, int tau_s, int tau_t,
-                                               const SceneNorms& nm, const DevParams& P,
-                                               float log2_scale) {
-  const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
-  const float dx = d2 > 0.0f ? d2 * rsqrtf(d2) : 0.0f;
-  const float tx = __log2f(1.0f + P.kappa * (dx * nm.x_rinv)) * log2_scale;
-  const int dt = tau_s - tau_t;
-  const float tt = dt > 0 ? (float)dt * nm.t_rinv : 0.0f;
-  return P.lambda_f * tf + P.lambda_x * tx + P.lambda_tau * tt;
+// FST cost of one pair (Eq. fst_cost) for the tensor-core path, with the
+// weights and normalisers folded into per-scene constants:
+//   C = kB - kA cos + kL log2(1 + kK d) + kT max(tau_s - tau_t, 0)
+// (kA = lambda_f / M_f, kB = kA (1 - min d_f), kK = kappa / M_x,
+// kL = lambda_x / log2(1 + kappa), kT = lambda_tau / M_tau); the distance
+// d = d2 rsqrt(d2) with d2 kept above 1e-30 (d = 0 gives log2(1) = 0), and
+// log2 from __log2f: within ~1e-6 of the plain formula, far inside the bf16
+// parity bar, and C(t, t) = 0 exactly.
+struct FstConst {
+  float kA, kB, kK, kL, kT;
+};
+__device__ __forceinline__ FstConst fst_const(const SceneNorms& nm, const DevParams& P) {
+  FstConst k;
+  k.kA = P.lambda_f * nm.f_rinv;
+  k.kB = k.kA * (1.0f - nm.f_lo);
+  k.kK = P.kappa * nm.x_rinv;
+  k.kL = P.lambda_x * (0.69314718055994531f * P.inv_log1p_kappa);  // log(1+x) = ln2 log2(1+x)
+  k.kT = P.lambda_tau * nm.t_rinv;
+  return k;
+}
+__device__ __forceinline__ float fst_cost_fold(const FstConst& k, float cosv, float dx, float dy,
+                                               float dz, float tau_s, float tau_t) {
+  const float d2 = fmaxf(fmaf(dz, dz, fmaf(dy, dy, dx * dx)), 1.0e-30f);
+  const float lg = __log2f(fmaf(k.kK, d2 * rsqrtf(d2), 1.0f));
+  return fmaf(k.kL, lg, fmaf(k.kT, fmaxf(tau_s - tau_t, 0.0f), fmaf(-k.kA, cosv, k.kB)));
 }
 
 // Warp-reduce a scene's running max / min cosine and merge it into stats.
@@ -221,29 +279,33 @@ __device__ __forceinline__ void flush_minmax(SceneStats* st, float cmax, float c
   }
 }
 
-// Tile t of the schedule -> (scene b, row tile I, column tile J).  MINMAX
-// visits only J >= I/2 (tiles holding a pair i <= j); COST visits all.
+// Unit p of the schedule -> (scene b, row tile I, column tile J): a unit is
+// a pair of row tiles (2P, 2P+1) and the cluster's CTA of rank c computes
+// I = 2P + c.  MINMAX visits only the tiles holding a pair i <= j (row tile
+// I needs J >= I/2, so a pair needs J >= P); COST visits all.
 template <int MODE>
-__device__ __forceinline__ void tile_coords(const TcArgs& a, int t, int& b, int& I, int& J) {
-  b = t / a.tiles_per_scene;
-  int r = t - b * a.tiles_per_scene;
+__device__ __forceinline__ void unit_coords(const TcArgs& a, int p, int cr, int& b, int& I,
+                                            int& J) {
+  b = p / a.pairs_per_scene;
+  int r = p - b * a.pairs_per_scene;
+  const int TP = (a.TI + 1) >> 1;
+  int P = 0;
   if (MODE == TC_COST) {
-    I = r / a.TJ;
-    J = r - I * a.TJ;
+    P = r / a.TJ;
+    J = r - P * a.TJ;
   } else {
-    I = 0;
-    while (r >= a.TJ - (I >> 1)) {
-      r -= a.TJ - (I >> 1);
-      ++I;
+    while (P < TP - 1 && r >= a.TJ - P) {
+      r -= a.TJ - P;
+      ++P;
     }
-    J = (I >> 1) + r;
+    J = P + r;
   }
+  I = 2 * P + cr;  // past the last row tile (odd TI): rows read as 0
 }
 
 template <int MODE>
 __global__ void __launch_bounds__(TC_THREADS, 1)
-    k_gram_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-              const TcArgs a) {
+    k_gram_tc(const __grid_constant__ CUtensorMap mapA, const TcArgs a) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[TC_STAGES], empty_bar[TC_STAGES];
   __shared__ __align__(8) uint64_t tfull_bar[2], tempty_bar[2];
@@ -252,12 +314,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t smem_base = (smem_u32(smem_raw) + 1023u) & ~1023u;  // 1024-B aligned ring
+  const int cr = (int)cluster_rank();                 // this CTA's row tile in the pair
+  const int cid = (int)(blockIdx.x >> 1), ncl = (int)(gridDim.x >> 1);
+  const uint16_t both = 0x3;
 
   if (threadIdx.x == 0) {
     s_abort = 0;
     for (int s = 0; s < TC_STAGES; ++s) {
       mbar_init(&full_bar[s], 1);   // producer's arrive + the TMA bytes
-      mbar_init(&empty_bar[s], 1);  // one tcgen05.commit
+      mbar_init(&empty_bar[s], 2);  // a tcgen05.commit from each CTA of the pair
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&tfull_bar[i], 1);     // one tcgen05.commit
@@ -265,7 +330,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
-    tma_prefetch_desc(&mapB);
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -277,6 +341,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  cluster_sync_all();  // both CTAs' barriers exist before either signals the other
   const uint32_t tmem_base = s_tmem_base;
 
   if (warp == 0) {
@@ -287,16 +352,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       uint32_t phase = 0;
       uint32_t pending = 0;        // stages holding a load not yet seen consumed
       uint32_t pend_parity = 0;    // parity of that load's full phase, per stage bit
-      for (int t = blockIdx.x; t < a.total_tiles && !s_abort; t += gridDim.x) {
+      for (int p = cid; p < a.total_pairs && !s_abort; p += ncl) {
         int b, I, J;
-        tile_coords<MODE>(a, t, b, I, J);
+        unit_coords<MODE>(a, p, cr, b, I, J);
         for (int kb = 0; kb < a.num_kb; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
           pending &= ~(1u << stage);
           const uint32_t sa = smem_base + (uint32_t)stage * TC_STAGE_BYTES;
           mbar_arrive_expect_tx(&full_bar[stage], TC_STAGE_BYTES);
           tma_load_3d(&mapA, &full_bar[stage], sa, kb * TC_BK, I * TC_BM, b, keep);
-          tma_load_3d(&mapB, &full_bar[stage], sa + TC_A_BYTES, kb * TC_BK, J * TC_BN, b, keep);
+          // own half of B into both CTAs; the peer's half arrives too
+          tma_load_3d_mc(&mapA, &full_bar[stage], sa + TC_A_BYTES + (uint32_t)cr * TC_A_BYTES,
+                         kb * TC_BK, J * TC_BN + cr * TC_BM, b, both, keep);
           pending |= 1u << stage;
           pend_parity = (pend_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == TC_STAGES) {
@@ -312,6 +379,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           if (pending & (1u << s))
             while (!mbar_test(&full_bar[s], (pend_parity >> s) & 1u) && globaltimer_ns() < drain) {
             }
+      } else {
+        // every stage released by both MMAs: the peer's last commits to this
+        // CTA's barriers have landed before the final cluster barrier
+        for (int i = 0; i < TC_STAGES; ++i) {
+          if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
+          if (++stage == TC_STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
       }
     }
   } else if (warp == 1) {
@@ -323,7 +400,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       uint32_t acc_phase = 0;
       uint64_t* last_commit = nullptr;
       uint32_t last_parity = 0;
-      for (int t = blockIdx.x; t < a.total_tiles && !s_abort; t += gridDim.x) {
+      for (int p = cid; p < a.total_pairs && !s_abort; p += ncl) {
         if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
         tc_fence_after();
         const uint32_t tmem_d = tmem_base + (uint32_t)(acc * TC_BN);
@@ -340,7 +417,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           for (int k = 0; k < TC_BK / 16; ++k)  // 32 bytes further along K per step
             umma_bf16(tmem_d, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k),
                       (kb > 0 || k > 0) ? 1u : 0u);
-          umma_commit(&empty_bar[stage]);  // frees the stage when these MMAs finish
+          umma_commit_mc(&empty_bar[stage], both);  // frees the stage (in both CTAs)
           last_commit = &empty_bar[stage];
           last_parity = phase;
           if (++stage == TC_STAGES) {
@@ -374,14 +451,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                                           TC_STAGES * TC_STAGE_BYTES) +
                  ew * TC_STG_FLOATS;               // this warp's 32 x 32 staging tile
     float4* s_col = reinterpret_cast<float4*>(stg);  // chunk columns: (x, y, z, 1/||f||)
-    int* s_tau = reinterpret_cast<int*>(stg + 4 * 32);  // ... and their frames
-    const float log2_scale = 0.69314718055994531f * a.P.inv_log1p_kappa;
+    float* s_tau = stg + 4 * 32;                        // ... their frames (exact floats)
+    float* s_vc = stg + 5 * 32;                         // ... and capacities (g0 only)
     const uint64_t stream_out = l2_policy_evict_first();
     int acc = 0;
     uint32_t acc_phase = 0;
     float cmax = -INFINITY, cmin = INFINITY;
     int cur_b = -1;
-    for (int t = blockIdx.x; t < a.total_tiles; t += gridDim.x) {
+    for (int p = cid; p < a.total_pairs; p += ncl) {
       // lane 0 waits, the warp follows it (keeps the warp converged for the
       // .sync.aligned TMEM loads below)
       int ok = 1;
@@ -390,7 +467,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       int b, I, J;
-      tile_coords<MODE>(a, t, b, I, J);
+      unit_coords<MODE>(a, p, cr, b, I, J);
       if (MODE == TC_MINMAX && b != cur_b) {
         if (cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
         cur_b = b;
@@ -401,13 +478,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const bool row_ok = gi < a.N;
       const size_t sb = (size_t)b * a.N;
       float4 ti = make_float4(0.f, 0.f, 0.f, 0.f);
-      int taui = 0;
+      float taui = 0.0f;
       if (row_ok) {
         ti = __ldg(a.tok + sb + gi);
-        if (MODE == TC_COST) taui = __ldg(a.frame + sb + gi);
+        if (MODE == TC_COST) taui = (float)__ldg(a.frame + sb + gi);
       }
-      SceneNorms nm;
-      if (MODE == TC_COST) nm = a.norms[b];
+      FstConst kf{};
+      if (MODE == TC_COST) kf = fst_const(a.norms[b], a.P);
+      float g0part = 0.0f;  // this row's first-gain terms over the warp's columns
       const uint32_t row_taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN);
 #pragma unroll 1
       for (int c = half * 4; c < half * 4 + 4; ++c) {
@@ -416,14 +494,17 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         {
           const int jl = j0 + lane;
           float4 tj = make_float4(0.f, 0.f, 0.f, 0.f);
-          int tauj = 0;
+          float tauj = 0.0f;
+          float vj = 0.0f;
           if (jl < a.N) {
             tj = __ldg(a.tok + sb + jl);
-            if (MODE == TC_COST) tauj = __ldg(a.frame + sb + jl);
+            if (MODE == TC_COST) tauj = (float)__ldg(a.frame + sb + jl);
+            if (MODE == TC_COST && a.g0) vj = __ldg(a.v + sb + jl);
           }
           __syncwarp();  // the previous chunk's staging reads are done
           s_col[lane] = tj;
           s_tau[lane] = tauj;
+          s_vc[lane] = vj;
           __syncwarp();
         }
         uint32_t v[32];
@@ -440,6 +521,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 cmin = fminf(cmin, cv);
               }
             }
+          } else if (j0 + 32 <= a.N && (j0 >= I * TC_BM + q * 32 + 32 || j0 + 32 <= I * TC_BM + q * 32)) {
+            // an interior chunk: every column is a token and none is a row
+            // of this warp, so no diagonal and no padding
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const float4 tj = s_col[e];
+              const float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * tj.w);
+              const float out =
+                  fst_cost_fold(kf, cv, ti.x - tj.x, ti.y - tj.y, ti.z - tj.z, taui, s_tau[e]);
+              if (a.g0) g0part = __fmaf_rn(s_vc[e], fmaxf(__fsub_rn(a.m0, out), 0.0f), g0part);
+              v[e] = __float_as_uint(out);
+            }
           } else {
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
@@ -448,10 +541,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               if (j < a.N) {
                 const float4 tj = s_col[e];
                 float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * tj.w);
-                if (j == gi && ti.w > 0.0f) cv = 1.0f;
-                const float dx = ti.x - tj.x, dy = ti.y - tj.y, dz = ti.z - tj.z;
-                const float d2 = dx * dx + dy * dy + dz * dz;
-                out = fst_cost_fast(cv, d2, taui, s_tau[e], nm, a.P, log2_scale);
+                if (j == gi && ti.w > 0.0f) cv = 1.0f;  // cos(f, f) = 1 exactly
+                out = fst_cost_fold(kf, cv, ti.x - tj.x, ti.y - tj.y, ti.z - tj.z, taui, s_tau[e]);
+                if (a.g0) g0part = __fmaf_rn(s_vc[e], fmaxf(__fsub_rn(a.m0, out), 0.0f), g0part);
               }
               v[e] = __float_as_uint(out);
             }
@@ -489,6 +581,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
         }
       }
+      if (MODE == TC_COST && a.g0 && row_ok)
+        a.g0[((size_t)b * (2 * a.TJ) + (size_t)(2 * J + half)) * a.N + gi] = g0part;
       tc_fence_before();
       mbar_arrive(&tempty_bar[acc]);  // accumulator free for the MMA warp
       if (++acc == 2) {
@@ -507,6 +601,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                  "r"(TC_TMEM_COLS)
                  : "memory");
   }
+  cluster_sync_all();  // neither CTA leaves while the other may still signal it
 }
 
 }  // namespace
@@ -567,12 +662,12 @@ int make_feature_map(CUtensorMap* map, const void* feats, int64_t B, int64_t N, 
 template <int MODE>
 int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const SceneNorms* norms,
               const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
-              SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s) {
+              SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s,
+              const float* v = nullptr, float* g0 = nullptr) {
   DeviceInfo di;
   if (device_info(&di) != CP_OK) return CP_ECUDA;
-  alignas(64) CUtensorMap mapA, mapB;
+  alignas(64) CUtensorMap mapA;  // 64 x 128 boxes: A tiles and the halves of B tiles
   CP_TRY_STATUS(make_feature_map(&mapA, feats, B, N, D, TC_BM));
-  CP_TRY_STATUS(make_feature_map(&mapB, feats, B, N, D, TC_BN));
   TcArgs a{};
   a.tok = tok;
   a.frame = frame;
@@ -581,6 +676,9 @@ int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const 
   a.cost = cost;
   a.ldc = ldc;
   a.vec_ok = (ldc % 4 == 0) && (reinterpret_cast<uintptr_t>(cost) % 16 == 0);
+  a.v = v;
+  a.g0 = g0;
+  a.m0 = P.m0;
   a.stats = stats;
   a.status = status;
   a.N = (int)N;
@@ -588,25 +686,38 @@ int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const 
   a.TI = (int)((N + TC_BM - 1) / TC_BM);
   a.TJ = (int)((N + TC_BN - 1) / TC_BN);
   a.num_kb = (int)((D + TC_BK - 1) / TC_BK);
-  int64_t tps = 0;
-  if (MODE == TC_COST) {
-    tps = (int64_t)a.TI * a.TJ;
-  } else {
-    for (int I = 0; I < a.TI; ++I) tps += a.TJ - (I >> 1);
-  }
-  const int64_t total = tps * B;
+  const int TP = (a.TI + 1) / 2;  // row-tile pairs (TP == TJ)
+  int64_t ups = 0;                // units per scene
+  if (MODE == TC_COST)
+    ups = (int64_t)TP * a.TJ;
+  else
+    for (int P2 = 0; P2 < TP; ++P2) ups += a.TJ - P2;
+  const int64_t total = ups * B;
   if (total > INT_MAX) return CP_EUNSUPPORTED;
-  a.tiles_per_scene = (int)tps;
-  a.total_tiles = (int)total;
+  a.pairs_per_scene = (int)ups;
+  a.total_pairs = (int)total;
   a.timeout_ns = timeout_ns;
-  const int grid = (int)(total < di.sm_count ? total : di.sm_count);
   auto fn = k_gram_tc<MODE>;
   if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)TC_SMEM),
                   "launch_gram_tc: smem attribute") != CP_OK)
     return CP_ECUDA;
-  fn<<<grid, TC_THREADS, TC_SMEM, s>>>(mapA, mapB, a);
-  return last_launch_status();
+  const int64_t clusters = total < di.sm_count / 2 ? total : di.sm_count / 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(2 * clusters));
+  cfg.blockDim = dim3(TC_THREADS);
+  cfg.dynamicSmemBytes = TC_SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, fn, mapA, a);
+  note_launch();
+  return cuda_status(e, "launch_gram_tc");
 }
 
 }  // namespace
@@ -620,9 +731,10 @@ int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64
 
 int launch_cost_tc(const void* feats, const float4* tok, const int32_t* frame,
                    const SceneNorms* norms, const DevParams& P, int64_t B, int64_t N, int64_t D,
-                   float* cost, int64_t ldc, int* status, uint64_t timeout_ns, cudaStream_t s) {
+                   float* cost, int64_t ldc, const float* v, float* g0, int* status,
+                   uint64_t timeout_ns, cudaStream_t s) {
   return launch_tc<TC_COST>(feats, tok, frame, norms, P, B, N, D, cost, ldc, nullptr, status,
-                            timeout_ns, s);
+                            timeout_ns, s, v, g0);
 }
 
 }  // namespace cp

@@ -120,7 +120,8 @@ int launch_finalize_norms(const SceneStats* stats, int64_t B, SceneNorms* norms,
 int launch_cost(const void* feats, int dtype, const float* inv, const float4* tok,
                 const float* pos, const int32_t* frame, const SceneNorms* norms,
                 const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
-                int* status, cudaStream_t s);
+                int* status, cudaStream_t s, const float* v = nullptr,
+                float* g0 = nullptr);
 // K4: capacity score r and capacity v (Eqs. fst_capacity_score, fst_capacity).
 int launch_capacity(const void* feats, int dtype, const float* inv, const float* pos,
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
@@ -133,7 +134,7 @@ int launch_slab(const float* cost, int64_t ldc, const int32_t* nbr, const DevPar
 int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
                int32_t* order32, float* gains, double* objective, uint64_t* partials,
-               uint32_t* counters, int* status, cudaStream_t s);
+               uint32_t* counters, int* status, cudaStream_t s, const float* g0 = nullptr);
 // Sort the B rows of K int32 indices ascending into int64 (and copy the
 // unsorted order out as int64 if order64 != NULL).
 int launch_sort_kept(const int32_t* idx32, int64_t B, int64_t K, int64_t* kept,

@@ -629,6 +629,8 @@ __device__ __forceinline__ unsigned long long untag_key(unsigned long long h, in
 struct LzClArgs {
   const float* cost;   // [B][N][ldc]
   const float* v;      // [B][N]
+  const float* g0;     // [B][g0_slots][N] first-gain partials from the cost epilogue, or null
+  int g0_slots;
   int32_t* order32;    // [B][K]
   float* gains;        // [B][K] or null
   double* objective;   // [B] or null
@@ -688,7 +690,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   }
   for (int i = threadIdx.x; i < a.nwords; i += LZ_THREADS) {
     chosen[i] = 0u;
-    fresh[i] = ~0u;  // step 0: every gain below is exact
+    fresh[i] = a.g0 ? 0u : ~0u;  // step 0: exact gains from the sweep below, or bounds
   }
   if (threadIdx.x < 3) {
     s_stats[threadIdx.x] = 0ull;
@@ -701,8 +703,25 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   }
   hw_cluster_sync();  // every block initialised before any peer writes to it
 
-  // step 0: every own candidate's gain exactly, one warp per row
-  for (int tl = w; tl < nown; tl += LZ_WARPS) {
+  if (a.g0) {
+    // step 0 from the cost epilogue's partial row sums: the same terms as
+    // the gain (exact products v d, each fused into a rounded sum), summed
+    // in another order, so like the gain within gamma_(n-1) =
+    // (n-1)u / (1 - (n-1)u) of the exact sum (u = 2^-24, n <= 16384 terms:
+    // the two differ by a factor below 1 + 2^-9); scaled by 1 + 2^-8 and
+    // rounded up they bound the gain, and are marked stale
+    const float* g0 = a.g0 + (size_t)(blockIdx.x >> lgC) * a.g0_slots * a.N;
+    for (int tl = threadIdx.x; tl < nown; tl += LZ_THREADS) {
+      const int t = (tl << lgC) | (int)crank;
+      float sum = 0.0f;
+      for (int sl = 0; sl < a.g0_slots; ++sl) sum = __fadd_rn(sum, g0[(size_t)sl * a.N + t]);
+      ub[tl] = __fmaf_ru(fmaxf(sum, 0.0f), 1.00390625f, 1.0e-30f);
+      if (a.use_mask)
+        for (int qq = 0; qq < 4; ++qq) nzm[4 * tl + qq] = (uint16_t)0xFFFFu;
+    }
+  }
+  // step 0 otherwise: every own candidate's gain exactly, one warp per row
+  for (int tl = a.g0 ? nown : w; tl < nown; tl += LZ_WARPS) {
     const float* crow = Cb + (size_t)((tl << lgC) | (int)crank) * a.ldc;
     float g0;
     if (a.use_mask) {
@@ -996,7 +1015,7 @@ static int cluster_size_for(int64_t B, int sm_count) {
 static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* v,
                                    const DevParams& P, int64_t B, int64_t N, int64_t K,
                                    int32_t* order32, float* gains, double* objective, int* status,
-                                   cudaStream_t s) {
+                                   cudaStream_t s, const float* g0) {
   DeviceInfo di;
   if (device_info(&di) != CP_OK) return CP_ECUDA;
   auto fn = k_sgs_lazy_cl;
@@ -1004,6 +1023,8 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
     LzClArgs a{};
     a.cost = cost;
     a.v = v;
+    a.g0 = g0;
+    a.g0_slots = (int)(2 * ((N + 255) / 256));
     a.order32 = order32;
     a.gains = gains;
     a.objective = objective;
@@ -1063,12 +1084,13 @@ template <bool LOCAL>
 static int sgs_lazy_launch(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                            const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
                            int32_t* order32, float* gains, double* objective, int* status,
-                           cudaStream_t s) {
+                           cudaStream_t s, const float* g0) {
   const int64_t ncols = LOCAL ? N : ldc;
   const size_t smem = sizeof(float) * (size_t)(2 * ncols + N) +
                       2 * sizeof(uint32_t) * (size_t)((N + 31) / 32);
   if (!LOCAL)
-    return sgs_lazy_cluster_launch(cost, ldc, v, P, B, N, K, order32, gains, objective, status, s);
+    return sgs_lazy_cluster_launch(cost, ldc, v, P, B, N, K, order32, gains, objective, status, s,
+                                   g0);
   auto fn = k_sgs_lazy<true>;
   if (smem > 48 * 1024 &&
       cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
@@ -1082,14 +1104,14 @@ static int sgs_lazy_launch(const float* cost, int64_t ldc, const float* slab, co
 int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
                int32_t* order32, float* gains, double* objective, uint64_t* partials,
-               uint32_t* counters, int* status, cudaStream_t s) {
+               uint32_t* counters, int* status, cudaStream_t s, const float* g0) {
   auto* part = reinterpret_cast<unsigned long long*>(partials);
   if (P.sgs_mode == 0) {
     if (P.g < N)
       return sgs_lazy_launch<true>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
-                                   status, s);
+                                   status, s, nullptr);
     return sgs_lazy_launch<false>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
-                                  status, s);
+                                  status, s, g0);
   }
   if (P.g < N)
     return sgs_launch_impl<true>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
