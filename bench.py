@@ -297,15 +297,15 @@ def run_ours(args, rank, world, local_rank, raw):
     value = whole_job_rate(B, world, ms_step)
 
     # roofline of the SGS kernel from its own events and its counted reads:
-    # the cost bytes its gain evaluations read (the kernel counts them: row
-    # blocks known to hold only zero terms are skipped) plus one row per
-    # step to update the coverage cost
+    # the cost bytes its gain evaluations and coverage updates read (the
+    # kernel counts them; row blocks known to hold only zero terms are
+    # skipped)
     hbm, tf_burst, tf_sust, peak_kind = measured_peaks()
     cstats = cp.coverprune_call_stats(ws)
     sgs_ms, sgs_launches = prof["sgs"]
     launches_per_step = max(sgs_launches // args.steps, 1)
     ldc = (N + 3) // 4 * 4
-    sgs_bytes_per_step = cstats["cost_bytes_read"] + B * K * N * 4
+    sgs_bytes_per_step = cstats["cost_bytes_read"]
     sgs_launch_ms = sgs_ms / max(sgs_launches, 1)
     sgs_gbs = (sgs_bytes_per_step / launches_per_step) / (sgs_launch_ms / 1000.0) / 1e9
     roofline_sgs = {"bound": "hbm", "kernel": "k_sgs_lazy<dense>", "achieved": round(sgs_gbs, 1),
@@ -361,7 +361,7 @@ def run_ours(args, rank, world, local_rank, raw):
     fprof = cp.coverprune_profile_read()
     fstats = cp.coverprune_call_stats(ws)
     f_ms = fprof["sgs"][0] / max(fprof["sgs"][1], 1)
-    f_bytes = fstats["cost_bytes_read"] + B * K * N * 4
+    f_bytes = fstats["cost_bytes_read"]
     f_gbs = f_bytes / (f_ms / 1000.0) / 1e9
     sweep = {"bound": "hbm", "kernel": "k_sgs<dense>", "achieved": round(f_gbs, 1), "peak": hbm,
              "unit": "GB/s", "frac": round(f_gbs / hbm, 4),

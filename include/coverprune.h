@@ -329,9 +329,11 @@ int coverprune_profile_read(double* ms, int64_t* launches, int n);
  *   rounds            decision rounds over all scenes and steps (lazy mode:
  *                     a step needs one or more; full sweep: one per step)
  *   cost_bytes_read   bytes of cost rows (or slab rows and their neighbour
- *                     indices) the gain evaluations read; the dense lazy
- *                     kernel skips row blocks whose terms are known to be
- *                     zero, so this can be well below gain_evaluations * 4N
+ *                     indices) the selection reads: every gain evaluation,
+ *                     and once per scene and step the winner's row for the
+ *                     coverage update; the dense lazy kernel skips row
+ *                     blocks whose terms are known to be zero, so this can
+ *                     be well below gain_evaluations * 4N
  * Returns CP_OK, CP_EINVAL or CP_ECUDA.
  */
 typedef struct {

@@ -240,6 +240,7 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
   const size_t nscenes = gridDim.x / cps;
   bool alive = true;
   unsigned long long my_evals = 0ull;  // rows this warp evaluated (lane 0 counts)
+  unsigned long long my_update_bytes = 0ull;  // coverage-update reads (thread 0 of block 0)
   for (int step = 0; step < K && alive; ++step) {
     unsigned long long best = 0ull;
     for (int t = gw; t < N; t += nw) {
@@ -299,6 +300,7 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
       if (c == 0) {
         order32[(size_t)b * K + step] = pick;
         if (gains) gains[(size_t)b * K + step] = s_gain;
+        my_update_bytes += LOCAL ? 8ull * (unsigned long long)P.g : 4ull * (unsigned long long)N;
       }
     }
     // S <- S u {t*} (Eq. sgs_update): lower the coverage cost of its targets
@@ -322,6 +324,7 @@ __global__ void __launch_bounds__(SGS_THREADS) k_sgs(
   if (c == 0 && threadIdx.x == 0) atomicAdd(&cstats[1], (unsigned long long)K);
   if (lane == 0 && my_evals)
     atomicAdd(&cstats[2], my_evals * (unsigned long long)(LOCAL ? 8 * P.g : 4 * ldc));
+  if (my_update_bytes) atomicAdd(&cstats[2], my_update_bytes);
   if (c == 0 && alive && objective) {
     const double F = objective_sum(sm_m, sm_v, N);
     if (threadIdx.x == 0) objective[b] = F;
@@ -414,6 +417,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
   __shared__ unsigned long long s_wkey[LZ_WARPS];
   __shared__ int s_wfresh[LZ_WARPS];
   unsigned long long my_evals = 0ull, my_rounds = 0ull;  // lane 0 / thread 0 count
+  unsigned long long my_update_bytes = 0ull;              // thread 0
 
   const int b = blockIdx.x;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -503,6 +507,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
       chosen[pick >> 5] |= 1u << (pick & 31);
       order32[(size_t)b * K + step] = pick;
       if (gains) gains[(size_t)b * K + step] = ub[pick];
+      my_update_bytes += LOCAL ? 8ull * (unsigned long long)P.g : 4ull * (unsigned long long)N;
     }
     // S <- S u {t*} (Eq. sgs_update)
     if (!LOCAL) {
@@ -525,6 +530,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
   if (threadIdx.x == 0) atomicAdd(&cstats[1], my_rounds);
   if (lane == 0 && my_evals)
     atomicAdd(&cstats[2], my_evals * (unsigned long long)(LOCAL ? 8 * P.g : 4 * ldc));
+  if (my_update_bytes) atomicAdd(&cstats[2], my_update_bytes);
   if (objective) {
     const double F = objective_sum(sm_m, sm_v, N);
     if (threadIdx.x == 0) objective[b] = F;
@@ -951,6 +957,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     const bool own = (pick & (a.C - 1)) == (int)crank;
     if (threadIdx.x == 0 && crank == 0) {
       const size_t o = (size_t)(blockIdx.x >> lgC) * a.K + step;
+      s_stats[2] += (unsigned long long)__popcll(WM) * (512ull << a.bit_shift);  // update reads
       a.order32[o] = pick;
       if (a.gains) a.gains[o] = __uint_as_float((uint32_t)(W >> 32));
     }
