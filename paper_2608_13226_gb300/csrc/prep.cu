@@ -522,7 +522,11 @@ __global__ void __launch_bounds__(1024) k_grid_build(const float* __restrict__ p
   }
 }
 
-// One thread per query token.
+// One thread per query token.  The KK best keys are kept unsorted with the
+// position of the worst: a closer point overwrites the worst (a select per
+// slot, so the list stays in registers) and the worst is found again; the
+// list is sorted once at the end.  Keys are (d^2 bits, index), as in the
+// brute-force kernels.
 template <int KK>
 __global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos, int N, int kk,
                                                   int gmax, const GridInfo* __restrict__ info,
@@ -538,9 +542,13 @@ __global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos,
   const float4* P = sorted + (size_t)b * N;
   const float qx = X[3 * j], qy = X[3 * j + 1], qz = X[3 * j + 2];
   const int cx = grid_coord(g, qx, 0), cy = grid_coord(g, qy, 1), cz = grid_coord(g, qz, 2);
+  // only the first kk slots are used; the others stay at the smallest key
+  // and never become the worst
   unsigned long long best[KK];
 #pragma unroll
-  for (int i = 0; i < KK; ++i) best[i] = ~0ull;
+  for (int i = 0; i < KK; ++i) best[i] = i < kk ? ~0ull : 0ull;
+  unsigned long long worst = ~0ull;
+  int wi = 0;
   const int rmax = max(g.dims[0], max(g.dims[1], g.dims[2]));
   for (int r = 0; r <= rmax; ++r) {
     for (int dz = -r; dz <= r; ++dz) {
@@ -554,39 +562,46 @@ __global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos,
           const int x = cx + dx;
           if (x < 0 || x >= g.dims[0]) continue;
           const int c = (z * g.dims[1] + y) * g.dims[0] + x;
-          for (int s = cs[c], e = cs[c + 1]; s < e; ++s) {
+          const int e = cs[c + 1];
+          for (int s = cs[c]; s < e; ++s) {
             const float4 p = P[s];
             const int k = __float_as_int(p.w);
             const uint32_t bits = __float_as_uint(sqdist_rn(qx, qy, qz, p.x, p.y, p.z));
-            if (k == j || bits > (uint32_t)(best[KK - 1] >> 32)) continue;
+            if (k == j || bits > (uint32_t)(worst >> 32)) continue;
             const unsigned long long key = ((unsigned long long)bits << 32) | (uint32_t)k;
-            if (key < best[KK - 1]) {
-              best[KK - 1] = key;
+            if (key >= worst) continue;
 #pragma unroll
-              for (int i = KK - 1; i > 0; --i)
-                if (best[i] < best[i - 1]) {
-                  const unsigned long long t = best[i];
-                  best[i] = best[i - 1];
-                  best[i - 1] = t;
-                }
-            }
+            for (int i = 0; i < KK; ++i) best[i] = i == wi ? key : best[i];
+            worst = 0ull;
+#pragma unroll
+            for (int i = 0; i < KK; ++i)
+              if (best[i] > worst) {
+                worst = best[i];
+                wi = i;
+              }
           }
         }
       }
     }
-    unsigned long long kth = ~0ull;  // the kk-th best key so far
-#pragma unroll
-    for (int i = 0; i < KK; ++i)
-      if (i == kk - 1) kth = best[i];
-    if (kth != ~0ull) {
+    if (worst != ~0ull) {  // the list is full: is anything closer still possible?
       const float reach = ((float)r - 1.0f / 1024.0f) * g.h;
-      if (reach > 0.0f && __uint_as_float((uint32_t)(kth >> 32)) < reach * reach) break;
+      if (reach > 0.0f && __uint_as_float((uint32_t)(worst >> 32)) < reach * reach) break;
     }
   }
+  // sort the kk keys ascending (the unused slots hold 0 and sort first)
+#pragma unroll
+  for (int i = 1; i < KK; ++i)
+#pragma unroll
+    for (int t = KK - 1; t >= i; --t)
+      if (best[t] < best[t - 1]) {
+        const unsigned long long x = best[t];
+        best[t] = best[t - 1];
+        best[t - 1] = x;
+      }
   int32_t* out = nbr + ((size_t)b * N + j) * kk;
 #pragma unroll
   for (int i = 0; i < KK; ++i)
-    if (i < kk) out[i] = (int32_t)(best[i] & 0xFFFFFFFFull);
+    if (i >= KK - kk) out[i - (KK - kk)] = (int32_t)(best[i] & 0xFFFFFFFFull);
 }
 
 // The largest pinned-fp32 squared distance over pairs, into stats.d2_max_bits:
