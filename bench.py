@@ -318,34 +318,52 @@ def run_ours(args, rank, world, local_rank, raw):
                     "rounds_per_step": cstats["rounds"],
                     "cost_bytes_read_per_step": cstats["cost_bytes_read"],
                     "full_sweep_evaluations_per_step": B * (K * N - K * (K - 1) // 2)}
-    def tflops(stage, flops_per_call):
+    def per_launch_ms(stage):
         ms, launches = prof[stage]
-        if ms <= 0 or launches <= 0:
-            return None
-        per_launch = flops_per_call * args.steps / launches
-        return per_launch / (ms / launches / 1000.0) / 1e12
+        return ms / launches if ms > 0 and launches > 0 else None
 
-    cost_tf = tflops("cost", B * 2.0 * N * N * D)            # full N x N x D product
-    gram_tf = tflops("gram", B * 1.0 * N * (N + 1) * D)      # the pairs i <= j once
-    roofline_gemm = {"bound": "tensor", "unit": "TFLOP/s", "peak": tf_burst,
-                     "cost_gemm": {"kernel": "k_gram_tc<COST>",
-                                   "achieved": cost_tf and round(cost_tf, 1),
-                                   "frac": cost_tf and round(cost_tf / tf_burst, 4),
-                                   "flops_per_launch": B * 2 * N * N * D,
-                                   "avg_launch_ms": round(prof["cost"][0] / max(prof["cost"][1], 1), 3)},
-                     "normaliser_gemm": {"kernel": "k_gram_tc<MINMAX>",
-                                         "achieved": gram_tf and round(gram_tf, 1),
-                                         "frac": gram_tf and round(gram_tf / tf_burst, 4),
-                                         "flops_per_launch": B * N * (N + 1) * D},
-                     "peak_source": peak_kind}
+    # the normaliser Gram (tensor cores): the pairs i <= j once, and it also
+    # stores every cosine, [B][N][ldc] fp32, for the elementwise cost pass
+    gram_ms = per_launch_ms("gram")
+    gram_launches_per_step = max(prof["gram"][1] // args.steps, 1)
+    gram_flops = B * N * (N + 1) * D // gram_launches_per_step
+    gram_tf = gram_flops / (gram_ms / 1000.0) / 1e12 if gram_ms else None
+    # the cost pass (HBM): reads the cosines and writes the cost in place,
+    # plus each scene's token, frame and capacity columns once
+    cost_ms = per_launch_ms("cost")
+    cost_launches_per_step = max(prof["cost"][1] // args.steps, 1)
+    cost_bytes = (2 * B * N * ldc * 4 + B * N * (16 + 4 + 4)) // cost_launches_per_step
+    cost_gbs = cost_bytes / (cost_ms / 1000.0) / 1e9 if cost_ms else None
+    roofline_front = {
+        "normaliser_gemm": {"bound": "tensor", "kernel": "k_gram_tc", "unit": "TFLOP/s",
+                            "achieved": gram_tf and round(gram_tf, 1), "peak": tf_burst,
+                            "frac": gram_tf and round(gram_tf / tf_burst, 4),
+                            "flops_per_launch": gram_flops,
+                            "cosine_bytes_stored_per_launch": B * N * ldc * 4
+                            // gram_launches_per_step,
+                            "avg_launch_ms": gram_ms and round(gram_ms, 3)},
+        "fst_cost": {"bound": "hbm", "kernel": "k_fst_apply", "unit": "GB/s",
+                     "achieved": cost_gbs and round(cost_gbs, 1), "peak": hbm,
+                     "frac": cost_gbs and round(cost_gbs / hbm, 4),
+                     "algorithmic_bytes_per_launch": cost_bytes,
+                     "traffic": read_traffic("k_fst_apply", cost_bytes),
+                     "avg_launch_ms": cost_ms and round(cost_ms, 3)},
+        "peak_source": peak_kind}
     # the line's roofline is the kernel with the largest share of the step
-    if prof["sgs"][0] >= prof["cost"][0]:
+    shares = {"sgs": prof["sgs"][0], "gram": prof["gram"][0], "cost": prof["cost"][0]}
+    top = max(shares, key=shares.get)
+    if top == "sgs":
         roofline = roofline_sgs
+    elif top == "gram":
+        r = roofline_front["normaliser_gemm"]
+        roofline = {"bound": "tensor", "kernel": r["kernel"], "achieved": r["achieved"],
+                    "peak": tf_burst, "unit": "TFLOP/s", "frac": r["frac"], "traffic": None,
+                    "peak_source": peak_kind, "algorithmic_flops_per_launch": gram_flops}
     else:
-        roofline = {"bound": "tensor", "kernel": "k_gram_tc<COST>", "achieved": round(cost_tf, 1),
-                    "peak": tf_burst, "unit": "TFLOP/s", "frac": round(cost_tf / tf_burst, 4),
-                    "traffic": None, "peak_source": peak_kind,
-                    "algorithmic_flops_per_launch": B * 2 * N * N * D}
+        r = roofline_front["fst_cost"]
+        roofline = {"bound": "hbm", "kernel": r["kernel"], "achieved": r["achieved"],
+                    "peak": hbm, "unit": "GB/s", "frac": r["frac"], "traffic": r["traffic"],
+                    "peak_source": peak_kind, "algorithmic_bytes_per_launch": cost_bytes}
 
     # the full sweep (every gain every step), same picks: its HBM roofline
     prm_full = cp.Params(sgs_mode=1)
@@ -505,7 +523,7 @@ def run_ours(args, rank, world, local_rank, raw):
                                     f"{rank * B}..{rank * B + B - 1} per rank"},
             "latency_ms": round(latency_ms, 3),
             "lite": lite, "roofline": roofline, "roofline_sgs": roofline_sgs,
-            "roofline_gemm": roofline_gemm, "sgs_full_sweep": sweep,
+            "roofline_front": roofline_front, "sgs_full_sweep": sweep,
             "stages_ms": stages, "gpu_launches": gpu_launches, "e2e": e2e,
             "clocks": clocks, "cpu_baseline": cpu}
     print(json.dumps(line), flush=True)
@@ -515,11 +533,11 @@ def run_ours(args, rank, world, local_rank, raw):
 
 
 def read_traffic(kernel: str, algorithmic_bytes: int):
-    """DRAM bytes of one SGS launch, scaled from the committed ncu record of
-    that kernel (profiles/<kernel>_traffic.txt: its DRAM bytes per
-    algorithmic byte on a captured launch) by this launch's algorithmic
-    bytes; None when no record exists or the kernel source has changed
-    since the counters were taken."""
+    """DRAM bytes of one launch of `kernel`, scaled from the committed ncu
+    record of that kernel (profiles/<kernel>_traffic.txt: its DRAM bytes per
+    algorithmic byte on a captured launch, and the sources it was built
+    from) by this launch's algorithmic bytes; None when no record exists or
+    those sources have changed since the counters were taken."""
     import hashlib
     path = os.path.join(ROOT, "profiles", f"{kernel}_traffic.txt")
     try:
@@ -528,8 +546,9 @@ def read_traffic(kernel: str, algorithmic_bytes: int):
             if ":" in line and not line.startswith("#"):
                 k, v = line.split(":", 1)
                 rec[k.strip()] = v.strip()
+        files = rec.get("source_files", "sgs.cu common.cuh").split()
         src = b"".join(open(os.path.join(ROOT, "paper_2608_13226_gb300", "csrc", f), "rb").read()
-                       for f in ("sgs.cu", "common.cuh"))
+                       for f in files)
         if hashlib.sha256(src).hexdigest()[:16] != rec.get("source_sha256"):
             return None
         return round(float(rec["dram_bytes_per_algorithmic_byte"]) * algorithmic_bytes)

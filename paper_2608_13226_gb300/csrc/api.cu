@@ -22,11 +22,11 @@ int launch_cost_simt(const void* feats, int dtype, const float* inv, const float
                      int64_t N, int64_t D, float* cost, int64_t ldc, cudaStream_t s);
 int64_t sgs_partials_count(int64_t B, int64_t N);
 int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64_t N, int64_t D,
-                          SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s);
-int launch_cost_tc(const void* feats, const float4* tok, const int32_t* frame,
-                   const SceneNorms* norms, const DevParams& P, int64_t B, int64_t N, int64_t D,
-                   float* cost, int64_t ldc, const float* v, float* g0, int* status,
-                   uint64_t timeout_ns, cudaStream_t s);
+                          SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s,
+                          float* cos_out, int64_t ldc);
+int launch_fst_apply(float* cost, int64_t ldc, int64_t B, int64_t N, const float4* tok,
+                     const int32_t* frame, const SceneNorms* norms, const DevParams& P,
+                     const float* v, float* g0, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Stage timing and launch counting.
@@ -112,24 +112,25 @@ int device_info(DeviceInfo* out) {
 }
 
 // bf16 features: tcgen05 tensor cores; fp32 features: fp32 FMA tiles (TF32
-// would round the features to 10 mantissa bits).
+// would round the features to 10 mantissa bits).  cos_out (bf16 only; may
+// be null): every cosine stored [B][N][ldc] for the elementwise cost pass.
 int launch_gram_minmax(const void* feats, int dtype, const float* inv, const float4* tok,
                        int64_t B, int64_t N, int64_t D, SceneStats* stats, int* status,
-                       uint64_t timeout_ns, cudaStream_t s) {
+                       uint64_t timeout_ns, cudaStream_t s, float* cos_out, int64_t ldc) {
   if (dtype == CP_BF16)
-    return launch_gram_minmax_tc(feats, tok, B, N, D, stats, status, timeout_ns, s);
+    return launch_gram_minmax_tc(feats, tok, B, N, D, stats, status, timeout_ns, s, cos_out, ldc);
   return launch_gram_minmax_simt(feats, dtype, inv, B, N, D, stats, s);
 }
 
-// g0 (bf16 features only; may be null): every row's first greedy gain terms
-// summed in the cost epilogue per 128-column half tile, [B][g0_slots(N)][N].
+// fp32 features: the FST cost on the SIMT cores (bf16 features take the
+// stored cosines and launch_fst_apply instead).
 int launch_cost(const void* feats, int dtype, const float* inv, const float4* tok,
                 const float* pos, const int32_t* frame, const SceneNorms* norms,
                 const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
-                int* status, cudaStream_t s, const float* v, float* g0) {
+                cudaStream_t s) {
   if (dtype == CP_BF16) {
-    return launch_cost_tc(feats, tok, frame, norms, P, B, N, D, cost, ldc, v, g0, status,
-                          P.timeout_ns, s);
+    note_message("launch_cost: bf16 features take the stored-cosine cost pass");
+    return CP_EUNSUPPORTED;
   }
   return launch_cost_simt(feats, dtype, inv, pos, frame, norms, P, B, N, D, cost, ldc, s);
 }
@@ -201,9 +202,6 @@ struct Plan {
 
 static size_t align_up(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// Slots of the cost epilogue's first-gain partial sums per row: one per
-// 128-column half of a 256-column tile.
-static int64_t g0_slots(int64_t N) { return 2 * ((N + 255) / 256); }
 
 // Workspace of coverprune_knn: status block, scene statistics, the grid.
 static size_t knn_ws_bytes(int64_t B, int64_t N) {
@@ -242,7 +240,7 @@ static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d,
     if (d.g < N) pl->slab = take(sizeof(float) * BN * (size_t)d.g);
     pl->partials = take(sizeof(uint64_t) * (size_t)sgs_partials_count(B, N));
     pl->order32 = take(sizeof(int32_t) * (size_t)B * (size_t)K);
-    pl->g0 = take(sizeof(float) * BN * (size_t)g0_slots(N));
+    pl->g0 = take(sizeof(float) * BN * (size_t)fst_apply_slots(pl->ldc));
   } else if (op == CP_OP_LITE) {
     pl->perm = take(sizeof(int32_t) * BN);
     pl->prefix = take(sizeof(uint64_t) * BN);
@@ -279,9 +277,12 @@ static T* at(void* ws, size_t off) {
 
 // Stats, inverse norms, neighbours and normalisers: the shared front of
 // every entry point.
+// cos_out (bf16 features only, may be null): the normaliser pass also stores
+// every cosine there, [B][N][ldc], for launch_fst_apply.
 static int run_front(const void* feats, int dtype, const float* pos, const int32_t* frame,
                      int64_t B, int64_t N, int64_t D, const DevParams& d, const Plan& pl, void* ws,
-                     float* norms_out, cudaStream_t s) {
+                     float* norms_out, cudaStream_t s, float* cos_out = nullptr,
+                     int64_t ldc = 0) {
   int* status = at<int>(ws, pl.hdr);
   SceneStats* stats = at<SceneStats>(ws, pl.stats);
   {
@@ -301,7 +302,8 @@ static int run_front(const void* feats, int dtype, const float* pos, const int32
   {
     Stage st(CP_STAGE_GRAM, s);
     CP_TRY(launch_gram_minmax(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), B, N,
-                              D, stats, status, d.timeout_ns, s));
+                              D, stats, status, d.timeout_ns, s,
+                              dtype == CP_BF16 ? cos_out : nullptr, ldc));
   }
   Stage st(CP_STAGE_PREP, s);
   CP_TRY(launch_finalize_norms(stats, B, at<SceneNorms>(ws, pl.norms), norms_out, s));
@@ -426,12 +428,18 @@ int coverprune_cost(const void* feats, int dtype, const float* pos, const int32_
   Plan pl;
   CP_TRY(check_ws(CP_OP_COST, B, N, 0, d, ws, ws_bytes, &pl));
   cudaStream_t s = (cudaStream_t)stream;
-  CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, norms, s));
+  // bf16: the normaliser pass stores the cosines into the output, then one
+  // elementwise pass turns them into the cost
+  CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, norms, s, cost, N));
   const SceneNorms* nm = at<SceneNorms>(ws, pl.norms);
   if (cost) {
     Stage st(CP_STAGE_COST, s);
-    CP_TRY(launch_cost(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), pos, frame,
-                       nm, d, B, N, D, cost, N, at<int>(ws, pl.hdr), s));
+    if (dtype == CP_BF16)
+      CP_TRY(launch_fst_apply(cost, N, B, N, at<float4>(ws, pl.tok), frame, nm, d, nullptr,
+                              nullptr, s));
+    else
+      CP_TRY(launch_cost(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), pos, frame,
+                         nm, d, B, N, D, cost, N, s));
   }
   if (capacity) {
     Stage st(CP_STAGE_CAPACITY, s);
@@ -459,7 +467,8 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
   CP_TRY(check_ws(CP_OP_SELECT, B, N, K, d, ws, ws_bytes, &pl));
   cudaStream_t s = (cudaStream_t)stream;
   int* status = at<int>(ws, pl.hdr);
-  CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, nullptr, s));
+  float* C = at<float>(ws, pl.cost);
+  CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, nullptr, s, C, pl.ldc));
   const SceneNorms* nm = at<SceneNorms>(ws, pl.norms);
   const float* inv = at<float>(ws, pl.inv);
   const int32_t* nbr = at<int32_t>(ws, pl.nbr);
@@ -469,13 +478,15 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
     CP_TRY(launch_capacity(feats, dtype, inv, pos, frame, nm, nbr, d, B, N, D, at<float>(ws, pl.r),
                            v, nullptr, s));
   }
-  float* C = at<float>(ws, pl.cost);
-  // the dense lazy selection starts from bounds the cost epilogue sums
+  // the dense lazy selection starts from bounds the cost pass sums
   float* g0 = (dtype == CP_BF16 && d.g >= N && d.sgs_mode == 0) ? at<float>(ws, pl.g0) : nullptr;
   {
     Stage st(CP_STAGE_COST, s);
-    CP_TRY(launch_cost(feats, dtype, inv, at<float4>(ws, pl.tok), pos, frame, nm, d, B, N, D, C,
-                       pl.ldc, status, s, v, g0));
+    if (dtype == CP_BF16)
+      CP_TRY(launch_fst_apply(C, pl.ldc, B, N, at<float4>(ws, pl.tok), frame, nm, d, v, g0, s));
+    else
+      CP_TRY(launch_cost(feats, dtype, inv, at<float4>(ws, pl.tok), pos, frame, nm, d, B, N, D, C,
+                         pl.ldc, s));
   }
   int32_t* order32 = at<int32_t>(ws, pl.order32);
   {

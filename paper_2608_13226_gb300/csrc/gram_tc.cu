@@ -1,22 +1,20 @@
 // K2/K3 for bf16 features on the 5th-generation tensor cores (tcgen05 + TMEM).
 //
 // The feature Gram G = F F^T of one scene is the method's only dense
-// contraction (the cosine of Eq. fst_metrics).  Two epilogues consume it:
-//   MINMAX  max and min of cos(f_i, f_j) over the pairs i <= j (the feature
-//           normaliser of Sec. 3.3) -- only the tiles on or above the
-//           diagonal run, no output but two atomics per warp
-//   COST    the FST cost of Eq. fst_cost, written row-major with stride ldc;
-//           optionally also every row's partial sums of v_j max(m0 - C(t,
-//           j), 0) over each 128-column half tile, one slot per half tile:
-//           the greedy's first gains, summed by the selection in another
-//           order than its own (it uses them inflated, as bounds)
+// contraction (the cosine of Eq. fst_metrics).  k_gram_tc computes it for
+// the pairs i <= j only (the tiles on or above the diagonal) and keeps the
+// max and min cosine (the feature normaliser of Sec. 3.3); with an output
+// buffer it also stores every cosine of a pair i <= j at [i][j] and at
+// [j][i].  The FST cost of Eq. fst_cost needs the normalisers of the whole
+// scene, so it follows as one elementwise pass over the stored cosines
+// (k_fst_apply, HBM-bound), which also sums the greedy's first gains.
 //
 // Persistent clusters of two CTAs (one CTA per SM).  The two CTAs of a
 // cluster compute the row tiles 2p and 2p+1 of the same 256-column tile:
 // each loads its own 128x64 A box and one 128-row half of the shared
 // 256x64 B box, multicast to both CTAs, so a CTA fetches 32 KB from L2 per
 // 64-deep step instead of 48 (measured: the normaliser GEMM 0.88 -> 0.95 of
-// the bf16 peak, the cost GEMM ~1% faster).  Each CTA has 10 warps:
+// the bf16 peak without the cosine stores).  Each CTA has 10 warps:
 //   warp 0      TMA producer: 128x64 bf16 boxes, 128-byte swizzle, into a
 //               4-stage shared-memory ring (48 KB a stage); a stage is
 //               refilled once both CTAs' MMAs have released it
@@ -25,12 +23,13 @@
 //               one of two 128x256 fp32 accumulators (double buffer)
 //   warps 2..9  epilogue: warps w and w+4 share TMEM lane quadrant w%4 and
 //               split the 256 columns; tcgen05.ld 32 lanes x 32 columns at a
-//               time, FST arithmetic in registers (or the min/max); the 32
-//               columns' token data is staged per warp in shared memory.
-//               Cost rows leave through a per-warp 32 x 32 shared-memory
-//               transpose (the same 4 KB that held the token data), so that
-//               each store instruction writes 4 rows x 128 contiguous bytes:
-//               whole L2 lines, which L2 takes without reading DRAM first
+//               time, cosines and their min/max in registers; the 32
+//               columns' inverse norms are staged per warp in shared memory.
+//               Chunks above the diagonal leave through a per-warp 32 x 32
+//               shared-memory transpose (the same 4 KB), so that each store
+//               instruction writes 4 rows x 128 contiguous bytes: whole L2
+//               lines, which L2 takes without reading DRAM first; their
+//               mirror images are column stores, one 128-byte line each
 // Stage hand-offs use mbarriers (a stage's "empty" barrier counts the
 // commits of both CTAs' MMA threads, multicast); the accumulator hand-off
 // uses tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
@@ -56,8 +55,6 @@ constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES +
                            (size_t)TC_EPI_WARPS * TC_STG_FLOATS * sizeof(float) +
                            1024;  // + alignment slack
 
-enum { TC_MINMAX = 0, TC_COST = 1 };
-
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16,
 // both K-major, M = 128, N = 256.
 constexpr uint32_t kIdesc = (1u << 4)              // D format: f32
@@ -68,15 +65,9 @@ constexpr uint32_t kIdesc = (1u << 4)              // D format: f32
 
 struct TcArgs {
   const float4* tok;      // [B*N] (x, y, z, 1/||f||)
-  const int32_t* frame;   // [B*N]
-  const SceneNorms* norms;
-  DevParams P;
-  float* cost;
+  float* cos_out;         // [B][N][ldc] every cosine, or null
   int64_t ldc;
-  int vec_ok;             // cost rows take 16-byte stores (ldc % 4 == 0, 16-byte base)
-  const float* v;         // [B*N] capacity, read when g0 is set
-  float* g0;              // [B][2 TJ][N] half-tile row sums of v_j max(m0 - C, 0), or null
-  float m0;
+  int vec_ok;             // cos_out rows take 16-byte stores (ldc % 4 == 0, 16-byte base)
   SceneStats* stats;
   int* status;
   int N, B, TI, TJ, num_kb;
@@ -167,6 +158,10 @@ __device__ __forceinline__ void tma_load_3d_mc(const CUtensorMap* map, uint64_t*
       "l"(policy)
       : "memory");
 }
+__device__ __forceinline__ void st_f32_policy(float* p, float v, uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" ::"l"(p), "f"(v), "l"(policy)
+               : "memory");
+}
 __device__ __forceinline__ void st_f4_policy(float* p, const float4& v, uint64_t policy) {
   asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x),
                "f"(v.y), "f"(v.z), "f"(v.w), "l"(policy)
@@ -240,33 +235,6 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// FST cost of one pair (Eq. fst_cost) for the tensor-core path, with the
-// weights and normalisers folded into per-scene constants:
-//   C = kB - kA cos + kL log2(1 + kK d) + kT max(tau_s - tau_t, 0)
-// (kA = lambda_f / M_f, kB = kA (1 - min d_f), kK = kappa / M_x,
-// kL = lambda_x / log2(1 + kappa), kT = lambda_tau / M_tau); the distance
-// d = d2 rsqrt(d2) with d2 kept above 1e-30 (d = 0 gives log2(1) = 0), and
-// log2 from __log2f: within ~1e-6 of the plain formula, far inside the bf16
-// parity bar, and C(t, t) = 0 exactly.
-struct FstConst {
-  float kA, kB, kK, kL, kT;
-};
-__device__ __forceinline__ FstConst fst_const(const SceneNorms& nm, const DevParams& P) {
-  FstConst k;
-  k.kA = P.lambda_f * nm.f_rinv;
-  k.kB = k.kA * (1.0f - nm.f_lo);
-  k.kK = P.kappa * nm.x_rinv;
-  k.kL = P.lambda_x * (0.69314718055994531f * P.inv_log1p_kappa);  // log(1+x) = ln2 log2(1+x)
-  k.kT = P.lambda_tau * nm.t_rinv;
-  return k;
-}
-__device__ __forceinline__ float fst_cost_fold(const FstConst& k, float cosv, float dx, float dy,
-                                               float dz, float tau_s, float tau_t) {
-  const float d2 = fmaxf(fmaf(dz, dz, fmaf(dy, dy, dx * dx)), 1.0e-30f);
-  const float lg = __log2f(fmaf(k.kK, d2 * rsqrtf(d2), 1.0f));
-  return fmaf(k.kL, lg, fmaf(k.kT, fmaxf(tau_s - tau_t, 0.0f), fmaf(-k.kA, cosv, k.kB)));
-}
-
 // Warp-reduce a scene's running max / min cosine and merge it into stats.
 __device__ __forceinline__ void flush_minmax(SceneStats* st, float cmax, float cmin) {
   for (int o = 16; o > 0; o >>= 1) {
@@ -281,29 +249,22 @@ __device__ __forceinline__ void flush_minmax(SceneStats* st, float cmax, float c
 
 // Unit p of the schedule -> (scene b, row tile I, column tile J): a unit is
 // a pair of row tiles (2P, 2P+1) and the cluster's CTA of rank c computes
-// I = 2P + c.  MINMAX visits only the tiles holding a pair i <= j (row tile
-// I needs J >= I/2, so a pair needs J >= P); COST visits all.
-template <int MODE>
+// I = 2P + c.  Only the tiles holding a pair i <= j are visited (row tile
+// I needs J >= I/2, so a pair needs J >= P).
 __device__ __forceinline__ void unit_coords(const TcArgs& a, int p, int cr, int& b, int& I,
                                             int& J) {
   b = p / a.pairs_per_scene;
   int r = p - b * a.pairs_per_scene;
   const int TP = (a.TI + 1) >> 1;
   int P = 0;
-  if (MODE == TC_COST) {
-    P = r / a.TJ;
-    J = r - P * a.TJ;
-  } else {
-    while (P < TP - 1 && r >= a.TJ - P) {
-      r -= a.TJ - P;
-      ++P;
-    }
-    J = P + r;
+  while (P < TP - 1 && r >= a.TJ - P) {
+    r -= a.TJ - P;
+    ++P;
   }
+  J = P + r;
   I = 2 * P + cr;  // past the last row tile (odd TI): rows read as 0
 }
 
-template <int MODE>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     k_gram_tc(const __grid_constant__ CUtensorMap mapA, const TcArgs a) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -354,7 +315,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       uint32_t pend_parity = 0;    // parity of that load's full phase, per stage bit
       for (int p = cid; p < a.total_pairs && !s_abort; p += ncl) {
         int b, I, J;
-        unit_coords<MODE>(a, p, cr, b, I, J);
+        unit_coords(a, p, cr, b, I, J);
         for (int kb = 0; kb < a.num_kb; ++kb) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
           pending &= ~(1u << stage);
@@ -450,9 +411,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     float* stg = reinterpret_cast<float*>(smem_raw + (smem_base - smem_u32(smem_raw)) +
                                           TC_STAGES * TC_STAGE_BYTES) +
                  ew * TC_STG_FLOATS;               // this warp's 32 x 32 staging tile
-    float4* s_col = reinterpret_cast<float4*>(stg);  // chunk columns: (x, y, z, 1/||f||)
-    float* s_tau = stg + 4 * 32;                        // ... their frames (exact floats)
-    float* s_vc = stg + 5 * 32;                         // ... and capacities (g0 only)
+    float* s_rn = stg;  // the chunk columns' 1/||f||
     const uint64_t stream_out = l2_policy_evict_first();
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -467,8 +426,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       int b, I, J;
-      unit_coords<MODE>(a, p, cr, b, I, J);
-      if (MODE == TC_MINMAX && b != cur_b) {
+      unit_coords(a, p, cr, b, I, J);
+      if (b != cur_b) {
         if (cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
         cur_b = b;
         cmax = -INFINITY;
@@ -477,84 +436,64 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const int gi = I * TC_BM + r;
       const bool row_ok = gi < a.N;
       const size_t sb = (size_t)b * a.N;
-      float4 ti = make_float4(0.f, 0.f, 0.f, 0.f);
-      float taui = 0.0f;
-      if (row_ok) {
-        ti = __ldg(a.tok + sb + gi);
-        if (MODE == TC_COST) taui = (float)__ldg(a.frame + sb + gi);
-      }
-      FstConst kf{};
-      if (MODE == TC_COST) kf = fst_const(a.norms[b], a.P);
-      float g0part = 0.0f;  // this row's first-gain terms over the warp's columns
+      const float rni = row_ok ? __ldg(a.tok + sb + gi).w : 0.0f;
+      const int r0 = I * TC_BM + q * 32;  // first row of this warp
       const uint32_t row_taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * TC_BN);
 #pragma unroll 1
       for (int c = half * 4; c < half * 4 + 4; ++c) {
         const int j0 = J * TC_BN + c * 32;
-        // stage the 32 columns' token data (one column per lane, coalesced)
+        // stage the 32 columns' inverse norms (one column per lane, coalesced)
         {
           const int jl = j0 + lane;
-          float4 tj = make_float4(0.f, 0.f, 0.f, 0.f);
-          float tauj = 0.0f;
-          float vj = 0.0f;
-          if (jl < a.N) {
-            tj = __ldg(a.tok + sb + jl);
-            if (MODE == TC_COST) tauj = (float)__ldg(a.frame + sb + jl);
-            if (MODE == TC_COST && a.g0) vj = __ldg(a.v + sb + jl);
-          }
+          const float rnj = jl < a.N ? __ldg(a.tok + sb + jl).w : 0.0f;
           __syncwarp();  // the previous chunk's staging reads are done
-          s_col[lane] = tj;
-          s_tau[lane] = tauj;
-          s_vc[lane] = vj;
+          s_rn[lane] = rnj;
           __syncwarp();
         }
         uint32_t v[32];
         tmem_ld32(row_taddr + (uint32_t)(c * 32), v);
         if (row_ok) {
-          if (MODE == TC_MINMAX) {
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const int j = j0 + e;
-              if (j < a.N) {
-                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * s_col[e].w);
-                if (j == gi && ti.w > 0.0f) cv = 1.0f;  // cos(f, f) = 1 exactly
-                cmax = fmaxf(cmax, cv);
-                cmin = fminf(cmin, cv);
-              }
+          for (int e = 0; e < 32; ++e) {
+            const int j = j0 + e;
+            float cv = 0.0f;  // pad columns N <= j < ldc hold 0
+            if (j < a.N) {
+              cv = clamp_cos(__uint_as_float(v[e]) * rni * s_rn[e]);
+              if (j == gi && rni > 0.0f) cv = 1.0f;  // cos(f, f) = 1 exactly
+              cmax = fmaxf(cmax, cv);
+              cmin = fminf(cmin, cv);
             }
-          } else if (j0 + 32 <= a.N && (j0 >= I * TC_BM + q * 32 + 32 || j0 + 32 <= I * TC_BM + q * 32)) {
-            // an interior chunk: every column is a token and none is a row
-            // of this warp, so no diagonal and no padding
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const float4 tj = s_col[e];
-              const float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * tj.w);
-              const float out =
-                  fst_cost_fold(kf, cv, ti.x - tj.x, ti.y - tj.y, ti.z - tj.z, taui, s_tau[e]);
-              if (a.g0) g0part = __fmaf_rn(s_vc[e], fmaxf(__fsub_rn(a.m0, out), 0.0f), g0part);
-              v[e] = __float_as_uint(out);
-            }
-          } else {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const int j = j0 + e;
-              float out = 0.0f;  // pad columns N <= j < ldc hold 0
-              if (j < a.N) {
-                const float4 tj = s_col[e];
-                float cv = clamp_cos(__uint_as_float(v[e]) * ti.w * tj.w);
-                if (j == gi && ti.w > 0.0f) cv = 1.0f;  // cos(f, f) = 1 exactly
-                out = fst_cost_fold(kf, cv, ti.x - tj.x, ti.y - tj.y, ti.z - tj.z, taui, s_tau[e]);
-                if (a.g0) g0part = __fmaf_rn(s_vc[e], fmaxf(__fsub_rn(a.m0, out), 0.0f), g0part);
-              }
-              v[e] = __float_as_uint(out);
-            }
+            v[e] = __float_as_uint(cv);
           }
         }
-        if (MODE == TC_COST) {
+        if (a.cos_out == nullptr) continue;
+        // a chunk wholly above the diagonal (every i < j) leaves through the
+        // transpose below, one crossing it row by row for j >= i; every
+        // i < j is also stored at [j][i] (lanes hold consecutive i, so each
+        // column is one 128-byte store)
+        const int where = j0 >= r0 + 31 ? 1 : (j0 + 31 < r0 ? -1 : 0);
+        if (where == 0 && row_ok) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const int j = j0 + e;
+            if (j >= gi && j < a.ldc)
+              a.cos_out[(sb + (size_t)gi) * (size_t)a.ldc + j] = __uint_as_float(v[e]);
+          }
+        }
+        if (where >= 0 && row_ok) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const int j = j0 + e;
+            if (j < a.N && gi < j)
+              st_f32_policy(a.cos_out + (sb + (size_t)j) * (size_t)a.ldc + gi,
+                            __uint_as_float(v[e]), stream_out);
+          }
+        }
+        if (where == 1) {
           // lane l writes row l's eight float4 chunks (chunk c at c ^ (l & 7),
           // so a phase of 8 lanes hits 8 distinct bank groups); store i (of
           // 8) then moves rows 4i + l/8, chunk l % 8: 4 rows x 128 bytes
-          const int r0 = I * TC_BM + q * 32;  // first row of this warp
-          __syncwarp();  // every lane is done with the token data
+          __syncwarp();  // every lane is done with the staged norms
 #pragma unroll
           for (int c = 0; c < 8; ++c)
             *reinterpret_cast<float4*>(stg + lane * 32 + 4 * (c ^ (lane & 7))) =
@@ -568,7 +507,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             const int grow = r0 + rr;
             const int col = j0 + 4 * c;
             if (grow < a.N && col < a.ldc) {
-              float* dst = a.cost + (sb + (size_t)grow) * (size_t)a.ldc + col;
+              float* dst = a.cos_out + (sb + (size_t)grow) * (size_t)a.ldc + col;
               if (a.vec_ok) {  // col % 4 == 0 and ldc % 4 == 0: the chunk fits
                 st_f4_policy(dst, val, stream_out);
               } else {
@@ -581,8 +520,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
         }
       }
-      if (MODE == TC_COST && a.g0 && row_ok)
-        a.g0[((size_t)b * (2 * a.TJ) + (size_t)(2 * J + half)) * a.N + gi] = g0part;
       tc_fence_before();
       mbar_arrive(&tempty_bar[acc]);  // accumulator free for the MMA warp
       if (++acc == 2) {
@@ -590,7 +527,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         acc_phase ^= 1u;
       }
     }
-    if (MODE == TC_MINMAX && cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
+    if (cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
   }
 
   tc_fence_before();
@@ -659,26 +596,20 @@ int make_feature_map(CUtensorMap* map, const void* feats, int64_t B, int64_t N, 
   return CP_OK;
 }
 
-template <int MODE>
-int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const SceneNorms* norms,
-              const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
-              SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s,
-              const float* v = nullptr, float* g0 = nullptr) {
+}  // namespace
+
+int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64_t N, int64_t D,
+                          SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s,
+                          float* cos_out, int64_t ldc) {
   DeviceInfo di;
   if (device_info(&di) != CP_OK) return CP_ECUDA;
   alignas(64) CUtensorMap mapA;  // 64 x 128 boxes: A tiles and the halves of B tiles
   CP_TRY_STATUS(make_feature_map(&mapA, feats, B, N, D, TC_BM));
   TcArgs a{};
   a.tok = tok;
-  a.frame = frame;
-  a.norms = norms;
-  a.P = P;
-  a.cost = cost;
+  a.cos_out = cos_out;
   a.ldc = ldc;
-  a.vec_ok = (ldc % 4 == 0) && (reinterpret_cast<uintptr_t>(cost) % 16 == 0);
-  a.v = v;
-  a.g0 = g0;
-  a.m0 = P.m0;
+  a.vec_ok = (ldc % 4 == 0) && (reinterpret_cast<uintptr_t>(cos_out) % 16 == 0);
   a.stats = stats;
   a.status = status;
   a.N = (int)N;
@@ -688,16 +619,13 @@ int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const 
   a.num_kb = (int)((D + TC_BK - 1) / TC_BK);
   const int TP = (a.TI + 1) / 2;  // row-tile pairs (TP == TJ)
   int64_t ups = 0;                // units per scene
-  if (MODE == TC_COST)
-    ups = (int64_t)TP * a.TJ;
-  else
-    for (int P2 = 0; P2 < TP; ++P2) ups += a.TJ - P2;
+  for (int P2 = 0; P2 < TP; ++P2) ups += a.TJ - P2;
   const int64_t total = ups * B;
   if (total > INT_MAX) return CP_EUNSUPPORTED;
   a.pairs_per_scene = (int)ups;
   a.total_pairs = (int)total;
   a.timeout_ns = timeout_ns;
-  auto fn = k_gram_tc<MODE>;
+  auto fn = k_gram_tc;
   if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)TC_SMEM),
                   "launch_gram_tc: smem attribute") != CP_OK)
@@ -720,21 +648,156 @@ int launch_tc(const void* feats, const float4* tok, const int32_t* frame, const 
   return cuda_status(e, "launch_gram_tc");
 }
 
-}  // namespace
+// ---------------------------------------------------------------------------
+// The FST cost from stored cosines, in place: C[i][j] = fst(cos[i][j], x, tau)
+// with the per-scene constants folded once (fst_const), and every row's
+// terms v_j max(m0 - C(i, j), 0) summed per 1024-column tile into
+// g0[b][tile][i] when g0 is given.
+// A block owns FA_COLS columns x FA_ROWS rows of one scene: each thread keeps
+// its four columns' token, frame and capacity in registers and walks the
+// rows, so the column data is read once per block (not once per element) and
+// every row of the tile is one contiguous 4 KB load and store.
+// ---------------------------------------------------------------------------
+namespace {
 
-int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64_t N, int64_t D,
-                          SceneStats* stats, int* status, uint64_t timeout_ns, cudaStream_t s) {
-  DevParams P{};
-  return launch_tc<TC_MINMAX>(feats, tok, nullptr, nullptr, P, B, N, D, nullptr, 0, stats, status,
-                              timeout_ns, s);
+// FST cost of one pair (Eq. fst_cost) with the weights and normalisers
+// folded into per-scene constants:
+//   C = kB - kA cos + kL log2(1 + kK d) + kT max(tau_s - tau_t, 0)
+// (kA = lambda_f / M_f, kB = kA (1 - min d_f), kK = kappa / M_x,
+// kL = lambda_x / log2(1 + kappa), kT = lambda_tau / M_tau); the distance
+// d = d2 rsqrt(d2) with d2 kept above 1e-30 (d = 0 gives log2(1) = 0), and
+// log2 from __log2f: within ~1e-6 of the plain formula, far inside the bf16
+// parity bar, and C(t, t) = 0 exactly.
+struct FstConst {
+  float kA, kB, kK, kL, kT;
+};
+__device__ __forceinline__ FstConst fst_const(const SceneNorms& nm, const DevParams& P) {
+  FstConst k;
+  k.kA = P.lambda_f * nm.f_rinv;
+  k.kB = k.kA * (1.0f - nm.f_lo);
+  k.kK = P.kappa * nm.x_rinv;
+  k.kL = P.lambda_x * (0.69314718055994531f * P.inv_log1p_kappa);  // log(1+x) = ln2 log2(1+x)
+  k.kT = P.lambda_tau * nm.t_rinv;
+  return k;
+}
+__device__ __forceinline__ float fst_cost_fold(const FstConst& k, float cosv, float dx, float dy,
+                                               float dz, float tau_s, float tau_t) {
+  const float d2 = fmaxf(fmaf(dz, dz, fmaf(dy, dy, dx * dx)), 1.0e-30f);
+  const float lg = __log2f(fmaf(k.kK, d2 * rsqrtf(d2), 1.0f));
+  return fmaf(k.kL, lg, fmaf(k.kT, fmaxf(tau_s - tau_t, 0.0f), fmaf(-k.kA, cosv, k.kB)));
 }
 
-int launch_cost_tc(const void* feats, const float4* tok, const int32_t* frame,
-                   const SceneNorms* norms, const DevParams& P, int64_t B, int64_t N, int64_t D,
-                   float* cost, int64_t ldc, const float* v, float* g0, int* status,
-                   uint64_t timeout_ns, cudaStream_t s) {
-  return launch_tc<TC_COST>(feats, tok, frame, norms, P, B, N, D, cost, ldc, nullptr, status,
-                            timeout_ns, s, v, g0);
+constexpr int FA_COLS = 1024, FA_ROWS = 32;
+
+template <bool VEC>
+__global__ void __launch_bounds__(256, 3)
+    k_fst_apply(float* __restrict__ cost, int64_t ldc, int N, const float4* __restrict__ tok,
+                const int32_t* __restrict__ frame, const SceneNorms* __restrict__ norms,
+                DevParams P, const float* __restrict__ v, float* __restrict__ g0) {
+  __shared__ float s_red[8][FA_ROWS];
+  const int b = blockIdx.z;
+  const int r0 = blockIdx.y * FA_ROWS;
+  const int j0 = blockIdx.x * FA_COLS + threadIdx.x * 4;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const size_t sb = (size_t)b * N;
+  const FstConst kf = fst_const(norms[b], P);
+  float4 tj[4];
+  float tauj[4], vj[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int j = j0 + u;
+    const bool in = j < N;
+    tj[u] = in ? __ldg(tok + sb + j) : make_float4(0.f, 0.f, 0.f, 0.f);
+    tauj[u] = in ? (float)__ldg(frame + sb + j) : 0.0f;
+    vj[u] = in && v ? __ldg(v + sb + j) : 0.0f;
+  }
+  const int nrow = min(FA_ROWS, N - r0);
+  for (int rr = 0; rr < nrow; rr += 4) {
+    float c[4][4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float* row = cost + (sb + (size_t)(r0 + rr + q)) * (size_t)ldc;
+      if (rr + q >= nrow) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) c[q][u] = 0.0f;
+      } else if (VEC) {
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (j0 < ldc) x = __ldcs(reinterpret_cast<const float4*>(row + j0));
+        c[q][0] = x.x, c[q][1] = x.y, c[q][2] = x.z, c[q][3] = x.w;
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) c[q][u] = j0 + u < ldc ? row[j0 + u] : 0.0f;
+      }
+    }
+    float p[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      p[q] = 0.0f;
+      if (rr + q >= nrow) continue;
+      const int i = r0 + rr + q;
+      const float4 ti = __ldg(tok + sb + i);
+      const float taui = (float)__ldg(frame + sb + i);
+      float o[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        o[u] = 0.0f;  // pad column
+        if (j0 + u < N) {
+          o[u] = fst_cost_fold(kf, c[q][u], ti.x - tj[u].x, ti.y - tj[u].y, ti.z - tj[u].z, taui,
+                               tauj[u]);
+          p[q] = __fmaf_rn(vj[u], fmaxf(__fsub_rn(P.m0, o[u]), 0.0f), p[q]);
+        }
+      }
+      float* row = cost + (sb + (size_t)i) * (size_t)ldc;
+      if (VEC) {
+        if (j0 < ldc)
+          __stcs(reinterpret_cast<float4*>(row + j0), make_float4(o[0], o[1], o[2], o[3]));
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (j0 + u < ldc) row[j0 + u] = o[u];
+      }
+    }
+    if (g0) {
+      // reduce-scatter the four rows' partials over the warp: lanes with
+      // bit 4 clear keep rows {0, 1}, set keep {2, 3}; then bit 3 picks one
+      // row; a butterfly over the low three bits completes each sum
+      const bool hb = lane & 16, mb = lane & 8;
+      const float k0 = hb ? p[2] : p[0], k1 = hb ? p[3] : p[1];
+      const float s0 = hb ? p[0] : p[2], s1 = hb ? p[1] : p[3];
+      const float q0 = k0 + __shfl_xor_sync(0xFFFFFFFFu, s0, 16);
+      const float q1 = k1 + __shfl_xor_sync(0xFFFFFFFFu, s1, 16);
+      float x = (mb ? q1 : q0) + __shfl_xor_sync(0xFFFFFFFFu, mb ? q0 : q1, 8);
+      x += __shfl_xor_sync(0xFFFFFFFFu, x, 4);
+      x += __shfl_xor_sync(0xFFFFFFFFu, x, 2);
+      x += __shfl_xor_sync(0xFFFFFFFFu, x, 1);
+      if ((lane & 7) == 0) s_red[w][rr + (hb ? 2 : 0) + (mb ? 1 : 0)] = x;
+    }
+  }
+  if (g0) {
+    __syncthreads();
+    if (threadIdx.x < nrow) {
+      float sum = s_red[0][threadIdx.x];
+#pragma unroll
+      for (int ww = 1; ww < 8; ++ww) sum += s_red[ww][threadIdx.x];
+      g0[((size_t)b * gridDim.x + blockIdx.x) * (size_t)N + r0 + threadIdx.x] = sum;
+    }
+  }
+}
+
+}  // namespace
+
+int fst_apply_slots(int64_t ldc) { return (int)((ldc + FA_COLS - 1) / FA_COLS); }
+
+int launch_fst_apply(float* cost, int64_t ldc, int64_t B, int64_t N, const float4* tok,
+                     const int32_t* frame, const SceneNorms* norms, const DevParams& P,
+                     const float* v, float* g0, cudaStream_t s) {
+  const bool vec = (ldc % 4 == 0) && (reinterpret_cast<uintptr_t>(cost) % 16 == 0);
+  dim3 grid((unsigned)fst_apply_slots(ldc), (unsigned)((N + FA_ROWS - 1) / FA_ROWS), (unsigned)B);
+  if (vec)
+    k_fst_apply<true><<<grid, 256, 0, s>>>(cost, ldc, (int)N, tok, frame, norms, P, v, g0);
+  else
+    k_fst_apply<false><<<grid, 256, 0, s>>>(cost, ldc, (int)N, tok, frame, norms, P, v, g0);
+  return last_launch_status();
 }
 
 }  // namespace cp

@@ -109,19 +109,20 @@ int launch_knn(const float* pos, const float4* tok, int64_t B, int64_t N, int kk
 // pairs into stats.
 int launch_gram_minmax(const void* feats, int dtype, const float* inv, const float4* tok,
                        int64_t B, int64_t N, int64_t D, SceneStats* stats, int* status,
-                       uint64_t timeout_ns, cudaStream_t s);
+                       uint64_t timeout_ns, cudaStream_t s,
+                       float* cos_out = nullptr, int64_t ldc = 0);
 // Scene diameter sqrt(max d^2) from stats into out[b].
 int launch_diameter(const SceneStats* stats, int64_t B, float* out, cudaStream_t s);
 // Normalisers from stats.  Optionally also the public [B, 6] float copy.
 int launch_finalize_norms(const SceneStats* stats, int64_t B, SceneNorms* norms,
                           float* norms_out, cudaStream_t s);
-// K3: the FST cost C[b][s][t] into cost + b*N*ldc + s*ldc + t for t < N;
-// columns N <= t < ldc are written as 0.
+// K3 for fp32 features: the FST cost C[b][s][t] into cost + b*N*ldc + s*ldc
+// + t for t < N; columns N <= t < ldc are written as 0.  (bf16 features:
+// launch_gram_minmax stores the cosines, then launch_fst_apply.)
 int launch_cost(const void* feats, int dtype, const float* inv, const float4* tok,
                 const float* pos, const int32_t* frame, const SceneNorms* norms,
                 const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
-                int* status, cudaStream_t s, const float* v = nullptr,
-                float* g0 = nullptr);
+                cudaStream_t s);
 // K4: capacity score r and capacity v (Eqs. fst_capacity_score, fst_capacity).
 int launch_capacity(const void* feats, int dtype, const float* inv, const float* pos,
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
@@ -130,6 +131,9 @@ int launch_capacity(const void* feats, int dtype, const float* inv, const float*
 // Local SGS: slab[b][t][k] = C(t, M_g(t)[k]) gathered from the dense cost.
 int launch_slab(const float* cost, int64_t ldc, const int32_t* nbr, const DevParams& P,
                 int64_t B, int64_t N, float* slab, cudaStream_t s);
+// Column tiles of the elementwise cost pass: the number of partial row sums
+// it writes per row into g0, [B][fst_apply_slots(ldc)][N].
+int fst_apply_slots(int64_t ldc);
 // K5: K greedy steps; order32[b*K + l] = token added at step l.
 int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,

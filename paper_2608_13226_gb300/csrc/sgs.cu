@@ -635,7 +635,7 @@ __device__ __forceinline__ unsigned long long untag_key(unsigned long long h, in
 struct LzClArgs {
   const float* cost;   // [B][N][ldc]
   const float* v;      // [B][N]
-  const float* g0;     // [B][g0_slots][N] first-gain partials from the cost epilogue, or null
+  const float* g0;     // [B][g0_slots][N] first-gain partial sums from the cost pass, or null
   int g0_slots;
   int32_t* order32;    // [B][K]
   float* gains;        // [B][K] or null
@@ -1031,7 +1031,7 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
     a.cost = cost;
     a.v = v;
     a.g0 = g0;
-    a.g0_slots = (int)(2 * ((N + 255) / 256));
+    a.g0_slots = fst_apply_slots(ldc);  // per column tile of the elementwise cost pass
     a.order32 = order32;
     a.gains = gains;
     a.objective = objective;
