@@ -428,10 +428,18 @@ int coverprune_cost(const void* feats, int dtype, const float* pos, const int32_
   Plan pl;
   CP_TRY(check_ws(CP_OP_COST, B, N, 0, d, ws, ws_bytes, &pl));
   cudaStream_t s = (cudaStream_t)stream;
-  // bf16: the normaliser pass stores the cosines into the output, then one
-  // elementwise pass turns them into the cost
+  // bf16: the normaliser pass stores the cosines into the output (the
+  // capacity reads its pairs there), then one elementwise pass turns them
+  // into the cost
   CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, norms, s, cost, N));
   const SceneNorms* nm = at<SceneNorms>(ws, pl.norms);
+  const float* cosines = dtype == CP_BF16 ? cost : nullptr;
+  if (capacity) {
+    Stage st(CP_STAGE_CAPACITY, s);
+    CP_TRY(launch_capacity(feats, dtype, at<float>(ws, pl.inv), pos, frame, nm,
+                           at<int32_t>(ws, pl.nbr), d, B, N, D, at<float>(ws, pl.r),
+                           at<float>(ws, pl.v), capacity, s, cosines, N));
+  }
   if (cost) {
     Stage st(CP_STAGE_COST, s);
     if (dtype == CP_BF16)
@@ -440,12 +448,6 @@ int coverprune_cost(const void* feats, int dtype, const float* pos, const int32_
     else
       CP_TRY(launch_cost(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), pos, frame,
                          nm, d, B, N, D, cost, N, s));
-  }
-  if (capacity) {
-    Stage st(CP_STAGE_CAPACITY, s);
-    CP_TRY(launch_capacity(feats, dtype, at<float>(ws, pl.inv), pos, frame, nm,
-                           at<int32_t>(ws, pl.nbr), d, B, N, D, at<float>(ws, pl.r),
-                           at<float>(ws, pl.v), capacity, s));
   }
   return CP_OK;
 }
@@ -476,7 +478,7 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
   {
     Stage st(CP_STAGE_CAPACITY, s);
     CP_TRY(launch_capacity(feats, dtype, inv, pos, frame, nm, nbr, d, B, N, D, at<float>(ws, pl.r),
-                           v, nullptr, s));
+                           v, nullptr, s, dtype == CP_BF16 ? C : nullptr, pl.ldc));
   }
   // the dense lazy selection starts from bounds the cost pass sums
   float* g0 = (dtype == CP_BF16 && d.g >= N && d.sgs_mode == 0) ? at<float>(ws, pl.g0) : nullptr;

@@ -48,6 +48,38 @@ __global__ void __launch_bounds__(256) k_capacity_r(
   if (lane == 0) r_all[(size_t)b * N + j] = P.n_cap > 0 ? acc / (float)P.n_cap : 0.0f;
 }
 
+// The same r_j from stored cosines: cos[b][j][k] (the normaliser Gram's
+// output, [B][N][ldc]) in place of the dot product, the rest identical.
+// One thread per token; its n gathers fall in one row, near its own index
+// (nearest neighbours sit in the same or adjacent frames).
+__global__ void __launch_bounds__(256) k_capacity_r_cos(
+    const float* __restrict__ cos_all, int64_t ldc, const float* __restrict__ pos_all,
+    const int32_t* __restrict__ frame_all, const SceneNorms* __restrict__ norms,
+    const int32_t* __restrict__ nbr_all, DevParams P, int N, float* __restrict__ r_all) {
+  const int j = blockIdx.x * 256 + threadIdx.x;
+  const int b = blockIdx.y;
+  if (j >= N) return;
+  const float* crow = cos_all + ((size_t)b * N + j) * (size_t)ldc;
+  const float* X = pos_all + (size_t)b * N * 3;
+  const int32_t* TAU = frame_all + (size_t)b * N;
+  const int32_t* nb = nbr_all + ((size_t)b * N + j) * P.kk;
+  const SceneNorms nm = norms[b];
+  const float xj = X[3 * j], yj = X[3 * j + 1], zj = X[3 * j + 2];
+  const int tj = TAU[j];
+  float acc = 0.0f;
+  for (int q = 0; q < P.n_cap; ++q) {
+    const int k = nb[q];
+    const float cosv = crow[k];
+    const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
+    const float dx = sqrtf(sqdist_rn(xj, yj, zj, X[3 * k], X[3 * k + 1], X[3 * k + 2]));
+    const float tx = (dx - nm.x_lo) * nm.x_rinv;
+    const int dt = tj - TAU[k];
+    const float tt = dt > 0 ? (float)dt * nm.t_rinv : 0.0f;
+    acc += P.alpha_f * tf + P.alpha_x * tx + P.alpha_tau * tt;
+  }
+  r_all[(size_t)b * N + j] = P.n_cap > 0 ? acc / (float)P.n_cap : 0.0f;
+}
+
 // v_j = r_j / sum_l r_l (phi = identity), uniform when the sum is 0 or the
 // uniform-capacity ablation is on.  One block per scene; the sum is taken in
 // fp64 in a fixed order.
@@ -81,9 +113,12 @@ __global__ void __launch_bounds__(1024) k_capacity_v(const float* __restrict__ r
 int launch_capacity(const void* feats, int dtype, const float* inv, const float* pos,
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
                     const DevParams& P, int64_t B, int64_t N, int64_t D, float* r, float* v,
-                    float* v_out, cudaStream_t s) {
+                    float* v_out, cudaStream_t s, const float* cos, int64_t ldc) {
   dim3 grid((unsigned)((N + 7) / 8), (unsigned)B);
-  if (dtype == CP_BF16)
+  if (cos)
+    k_capacity_r_cos<<<dim3((unsigned)((N + 255) / 256), (unsigned)B), 256, 0, s>>>(
+        cos, ldc, pos, frame, norms, nbr, P, (int)N, r);
+  else if (dtype == CP_BF16)
     k_capacity_r<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)feats, inv, pos, frame,
                                                       norms, nbr, P, (int)N, (int)D, r);
   else

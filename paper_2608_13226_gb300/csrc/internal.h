@@ -124,10 +124,13 @@ int launch_cost(const void* feats, int dtype, const float* inv, const float4* to
                 const DevParams& P, int64_t B, int64_t N, int64_t D, float* cost, int64_t ldc,
                 cudaStream_t s);
 // K4: capacity score r and capacity v (Eqs. fst_capacity_score, fst_capacity).
+// cos (may be null): every cosine, [B][N][ldc], as the normaliser pass
+// stores it; the pairs' cosines are then read from it, not recomputed.
 int launch_capacity(const void* feats, int dtype, const float* inv, const float* pos,
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
                     const DevParams& P, int64_t B, int64_t N, int64_t D, float* r, float* v,
-                    float* v_out, cudaStream_t s);
+                    float* v_out, cudaStream_t s, const float* cos = nullptr,
+                    int64_t ldc = 0);
 // Local SGS: slab[b][t][k] = C(t, M_g(t)[k]) gathered from the dense cost.
 int launch_slab(const float* cost, int64_t ldc, const int32_t* nbr, const DevParams& P,
                 int64_t B, int64_t N, float* slab, cudaStream_t s);

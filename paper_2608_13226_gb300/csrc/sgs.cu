@@ -45,33 +45,34 @@ __device__ __forceinline__ float gain_term(float acc, float v, float m, float c)
 }
 
 // Partial gain over quarter q of a dense padded row (ncols % 4 == 0, pad
-// v = 0): the row's float4 chunks are cut into four contiguous quarters;
-// lane l sums chunks l, l+32, ... of the quarter in ascending order, then a
-// butterfly (identical result in every lane).
+// v = 0).  The row's float4 chunks are taken in iterations of 32 (iteration
+// it: chunks 32 it .. 32 it + 31, 512 contiguous bytes) and quarter q owns
+// the iterations q, q + 4, q + 8, ...: a row's positive terms cluster by
+// token index (nearby tokens), and interleaving spreads them evenly over the
+// four quarters.  Lane l sums chunk 32 it + l of each owned iteration in
+// ascending order, then a butterfly (identical result in every lane).
 __device__ __forceinline__ float quarter_gain(const float* __restrict__ crow, const float* sm_m,
                                               const float* sm_v, int ncols, int q, int lane) {
   const float4* row = reinterpret_cast<const float4*>(crow);
   const float4* m4 = reinterpret_cast<const float4*>(sm_m);
   const float4* v4 = reinterpret_cast<const float4*>(sm_v);
   const int nq = ncols >> 2;
-  const int Q4 = (nq + 3) >> 2;
-  const int q_end = min(nq, (q + 1) * Q4);
   float acc = 0.0f;
-  int i = q * Q4 + lane;
-  for (; i + 224 < q_end; i += 256) {
+  int i = 32 * q + lane;
+  for (; i + 7 * 128 < nq; i += 8 * 128) {
     float4 cs[8];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) cs[u] = ld_stream_f4(row + i + 32 * u);
+    for (int u = 0; u < 8; ++u) cs[u] = ld_stream_f4(row + i + 128 * u);
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
-      const float4 mm = m4[i + 32 * u], vv = v4[i + 32 * u];
+      const float4 mm = m4[i + 128 * u], vv = v4[i + 128 * u];
       acc = gain_term(acc, vv.x, mm.x, cs[u].x);
       acc = gain_term(acc, vv.y, mm.y, cs[u].y);
       acc = gain_term(acc, vv.z, mm.z, cs[u].z);
       acc = gain_term(acc, vv.w, mm.w, cs[u].w);
     }
   }
-  for (; i < q_end; i += 32) {
+  for (; i < nq; i += 128) {
     const float4 c0 = ld_stream_f4(row + i);
     const float4 mm = m4[i], vv = v4[i];
     acc = gain_term(acc, vv.x, mm.x, c0.x);
@@ -87,9 +88,8 @@ __device__ __forceinline__ float combine_quarters(float s0, float s1, float s2, 
   return __fadd_rn(__fadd_rn(__fadd_rn(s0, s1), s2), s3);
 }
 
-// quarter_gain over the blocks a mask names.  Quarter q's float4 chunks are
-// visited in iterations of 32 (iteration u: chunks q*Q4 + 32u + lane); bit
-// u >> bit_shift of m16 says whether iteration u may hold a positive term.  An
+// quarter_gain over the blocks a mask names.  Quarter q's u-th iteration
+// holds chunks 32 (4u + q) + lane; bit u >> bit_shift of m16 says whether iteration u may hold a positive term.  An
 // iteration whose terms are all zero leaves every lane's sum unchanged (each
 // term is v * max(m - C, 0) = +0 and acc + 0 = acc), so skipping it returns
 // exactly quarter_gain's value.  A term stays zero once m <= C, because m
@@ -103,10 +103,8 @@ __device__ __forceinline__ float quarter_gain_masked(const float* __restrict__ c
   const float4* m4 = reinterpret_cast<const float4*>(sm_m);
   const float4* v4 = reinterpret_cast<const float4*>(sm_v);
   const int nq = ncols >> 2;
-  const int Q4 = (nq + 3) >> 2;
-  const int q0 = q * Q4;
-  const int q_end = min(nq, q0 + Q4);
-  const int nit = q_end > q0 ? (q_end - q0 + 31) >> 5 : 0;
+  const int NI = (nq + 31) >> 5;                    // iterations of the whole row
+  const int nit = NI > q ? (NI - q + 3) >> 2 : 0;   // ... owned by quarter q
   uint32_t todo = m16 & 0xFFFFu;
   if (bit_shift) {  // each bit covers two iterations: spread bit i to bits 2i, 2i+1
     todo = (todo | (todo << 8)) & 0x00FF00FFu;
@@ -129,15 +127,15 @@ __device__ __forceinline__ float quarter_gain_masked(const float* __restrict__ c
     float4 cs[8];
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
-      const int i = q0 + 32 * us[s] + lane;
-      cs[s] = (us[s] >= 0 && i < q_end) ? ld_stream_f4(row + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int i = 128 * us[s] + 32 * q + lane;
+      cs[s] = (us[s] >= 0 && i < nq) ? ld_stream_f4(row + i) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
       if (us[s] < 0) break;  // warp-uniform
-      const int i = q0 + 32 * us[s] + lane;
+      const int i = 128 * us[s] + 32 * q + lane;
       bool nz = false;
-      if (i < q_end) {
+      if (i < nq) {
         const float4 mm = m4[i], vv = v4[i];
         // d = max(m - C, 0) is +0 or positive, so the OR of the bit
         // patterns is zero iff all four terms are zero
@@ -875,14 +873,15 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
       if (kb != 0ull && kb != R) {
         const int t = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull));
         const int tl = t >> lgC;
-        const int nq = ncols >> 2, Q4 = (nq + 3) >> 2;
+        const int nq = ncols >> 2;
         const float4* row = reinterpret_cast<const float4*>(Cb + (size_t)t * a.ldc);
         for (int bb = lane; bb < 64; bb += 32) {
           if (!((nzm[4 * tl + (bb >> 4)] >> (bb & 15)) & 1u)) continue;
-          const int q0 = (bb >> 4) * Q4, q_end = min(nq, q0 + Q4);
-          const int i0 = q0 + (32 << a.bit_shift) * (bb & 15);
-          const int i1 = min(q_end, i0 + (32 << a.bit_shift));
-          if (i1 > i0) prefetch_l2(row + i0, (uint32_t)(16 * (i1 - i0)));
+          const int u0 = (bb & 15) << a.bit_shift, u1 = ((bb & 15) + 1) << a.bit_shift;
+          for (int u = u0; u < u1; ++u) {
+            const int i0 = 128 * u + 32 * (bb >> 4);  // iteration 4u + quarter
+            if (i0 < nq) prefetch_l2(row + i0, (uint32_t)(16 * min(32, nq - i0)));
+          }
         }
       }
     }
@@ -968,14 +967,13 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     {
       const float4* row = reinterpret_cast<const float4*>(Cb + (size_t)pick * a.ldc);
       float4* m4 = reinterpret_cast<float4*>(sm_m);
-      const int nq = ncols >> 2, Q4 = (nq + 3) >> 2;
+      const int nq = ncols >> 2;
       for (int bb = w; bb < 64; bb += LZ_WARPS) {
         if (!((WM >> bb) & 1ull)) continue;
-        const int q0 = (bb >> 4) * Q4, q_end = min(nq, q0 + Q4);
         const int u0 = (bb & 15) << a.bit_shift, u1 = ((bb & 15) + 1) << a.bit_shift;
         for (int u = u0; u < u1; ++u) {
-          const int i = q0 + 32 * u + lane;
-          if (i < q_end) {
+          const int i = 128 * u + 32 * (bb >> 4) + lane;  // iteration 4u + quarter
+          if (i < nq) {
             const float4 c = __ldg(row + i);
             float4 mm = m4[i];
             mm.x = fminf(mm.x, c.x);
@@ -1045,7 +1043,7 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
     a.lgC = C >= 8 ? 3 : C >= 4 ? 2 : C >= 2 ? 1 : 0;
     a.NC = (int)((N + C - 1) / C);
     a.nwords = (a.NC + 31) / 32;
-    const int nit_max = (int)(((ldc / 4 + 3) / 4 + 31) / 32);  // iterations per quarter
+    const int nit_max = (int)(((ldc / 4 + 31) / 32 + 3) / 4);  // iterations per quarter
     a.bit_shift = nit_max <= 16 ? 0 : 1;
     a.off_v = (uint32_t)(sizeof(float) * ldc);
     a.off_ub = (uint32_t)(sizeof(float) * 2 * ldc);
