@@ -250,19 +250,34 @@ __device__ __forceinline__ void flush_minmax(SceneStats* st, float cmax, float c
 // Unit p of the schedule -> (scene b, row tile I, column tile J): a unit is
 // a pair of row tiles (2P, 2P+1) and the cluster's CTA of rank c computes
 // I = 2P + c.  Only the tiles holding a pair i <= j are visited (row tile
-// I needs J >= I/2, so a pair needs J >= P).
+// I needs J >= I/2, so a pair needs J >= P).  A scene's units go in bands
+// of TC_BAND row-tile pairs, each band column by column (J ascending, then
+// P ascending), so the units in flight at once share a few A and B tiles
+// in L2 instead of sweeping every column tile of the scene.
+constexpr int TC_BAND = 8;
 __device__ __forceinline__ void unit_coords(const TcArgs& a, int p, int cr, int& b, int& I,
                                             int& J) {
   b = p / a.pairs_per_scene;
   int r = p - b * a.pairs_per_scene;
-  const int TP = (a.TI + 1) >> 1;
-  int P = 0;
-  while (P < TP - 1 && r >= a.TJ - P) {
-    r -= a.TJ - P;
-    ++P;
+  const int TP = (a.TI + 1) >> 1;  // == TJ
+  int P0 = 0, P1 = min(TC_BAND, TP) - 1;
+  for (;;) {  // the band holding unit r: columns J >= P0, min(J, P1) - P0 + 1 units each
+    const int hg = P1 - P0 + 1;
+    const int cnt = hg * (hg + 1) / 2 + (a.TJ - 1 - P1) * hg;
+    if (r < cnt || P1 >= TP - 1) break;
+    r -= cnt;
+    P0 += TC_BAND;
+    P1 = min(P0 + TC_BAND, TP) - 1;
   }
-  J = P + r;
-  I = 2 * P + cr;  // past the last row tile (odd TI): rows read as 0
+  int Jc = P0;
+  for (;;) {
+    const int h = min(Jc, P1) - P0 + 1;
+    if (r < h || Jc >= a.TJ - 1) break;
+    r -= h;
+    ++Jc;
+  }
+  J = Jc;
+  I = 2 * (P0 + r) + cr;  // past the last row tile (odd TI): rows read as 0
 }
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
@@ -666,8 +681,21 @@ namespace {
 // (kA = lambda_f / M_f, kB = kA (1 - min d_f), kK = kappa / M_x,
 // kL = lambda_x / log2(1 + kappa), kT = lambda_tau / M_tau); the distance
 // d = d2 rsqrt(d2) with d2 kept above 1e-30 (d = 0 gives log2(1) = 0), and
-// log2 from __log2f: within ~1e-6 of the plain formula, far inside the bf16
-// parity bar, and C(t, t) = 0 exactly.
+// log2 from the hardware approximation: within ~1e-6 of the plain formula,
+// far inside the bf16 parity bar, and C(t, t) = 0 exactly.  Both inputs are
+// normal floats (d2 >= 1e-30, 1 + kK d >= 1), where the flush-to-zero forms
+// of the two instructions return what the plain ones do, without their
+// subnormal-input handling.
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float rsqrt_approx(float x) {
+  float y;
+  asm("rsqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 struct FstConst {
   float kA, kB, kK, kL, kT;
 };
@@ -683,7 +711,7 @@ __device__ __forceinline__ FstConst fst_const(const SceneNorms& nm, const DevPar
 __device__ __forceinline__ float fst_cost_fold(const FstConst& k, float cosv, float dx, float dy,
                                                float dz, float tau_s, float tau_t) {
   const float d2 = fmaxf(fmaf(dz, dz, fmaf(dy, dy, dx * dx)), 1.0e-30f);
-  const float lg = __log2f(fmaf(k.kK, d2 * rsqrtf(d2), 1.0f));
+  const float lg = lg2_approx(fmaf(k.kK, d2 * rsqrt_approx(d2), 1.0f));
   return fmaf(k.kL, lg, fmaf(k.kT, fmaxf(tau_s - tau_t, 0.0f), fmaf(-k.kA, cosv, k.kB)));
 }
 
