@@ -19,6 +19,7 @@ cores on a bounded sample of the same workload, scaled to scenes per second.
 from __future__ import annotations
 
 import argparse
+import datetime
 import json
 import math
 import multiprocessing as mp
@@ -87,7 +88,7 @@ def measured_peaks():
 # clocks under load
 # --------------------------------------------------------------------------
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -95,6 +96,22 @@ class ClockSampler:
         self.index = index
         self.proc = None
         self.path = None
+        self.window = None  # (start, end) of the timed region, local wall time
+
+    def wait_first_sample(self, limit_s: float = 3.0):
+        """Returns once nvidia-smi has written a row (or after limit_s)."""
+        t0 = time.time()
+        while self.proc is not None and time.time() - t0 < limit_s:
+            try:
+                if os.path.getsize(self.path) > 0:
+                    return
+            except OSError:
+                return
+            time.sleep(0.02)
+
+    def mark(self, start: bool):
+        now = datetime.datetime.now()
+        self.window = (now, None) if start else (self.window[0] if self.window else now, now)
 
     def __enter__(self):
         fd, self.path = tempfile.mkstemp(suffix=".csv")
@@ -102,7 +119,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-i", str(self.index), "-lms", "200", "-f", self.path],
+                 "-i", str(self.index), "-lms", "50", "-f", self.path],
                 stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
@@ -121,7 +138,7 @@ class ClockSampler:
         try:
             for line in open(self.path):
                 parts = [p.strip() for p in line.split(",")]
-                if len(parts) >= 9:
+                if len(parts) >= 10:
                     rows.append(parts)
         except OSError:
             pass
@@ -130,17 +147,30 @@ class ClockSampler:
                 os.unlink(self.path)
             except OSError:
                 pass
+        # keep the samples taken inside the timed window (all, if none is)
+        inside = []
+        if self.window and self.window[1] is not None:
+            for r in rows:
+                try:
+                    t = datetime.datetime.strptime(r[0], "%Y/%m/%d %H:%M:%S.%f")
+                except ValueError:
+                    continue
+                if self.window[0] <= t <= self.window[1]:
+                    inside.append(r)
+        scope = "timed region" if inside else "whole sampler run"
+        rows = inside or rows
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
-        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
-        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
-        pw = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        pw = [float(r[4]) for r in rows if r[4].replace(".", "").isdigit()]
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        reasons = sorted({n for r in rows for n, v in zip(names, r[6:10]) if v.lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None,
                 "power_w_max": max(pw) if pw else None,
-                "reasons": reasons, "samples": len(rows)}
+                "reasons": reasons, "samples": len(rows), "scope": scope,
+                "interval_ms": 50}
 
 
 # --------------------------------------------------------------------------
@@ -274,19 +304,22 @@ def run_ours(args, rank, world, local_rank, raw):
     def max_over_ranks(x):
         return reduce_max(x, dist, dev)
 
-    for _ in range(args.warmup):
-        step()
-    barrier()
-    cp.coverprune_profile_read()  # clear
-    cp.coverprune_profile_enable(True)
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local_rank) as clk:
+        clk.wait_first_sample()
+        for _ in range(args.warmup):
+            step()
         barrier()
+        cp.coverprune_profile_read()  # clear
+        cp.coverprune_profile_enable(True)
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier()
+        clk.mark(True)
         ev0.record(stream)
         for _ in range(args.steps):
             step()
         ev1.record(stream)
         barrier()
+        clk.mark(False)
     cp.coverprune_profile_enable(False)
     prof = cp.coverprune_profile_read()
     clocks = clk.summary()
@@ -448,7 +481,7 @@ def run_ours(args, rank, world, local_rank, raw):
     inputs = [(torch.empty_like(feats), torch.empty_like(pos), torch.empty_like(fr))
               for _ in range(2)]
     copy_stream = torch.cuda.Stream()
-    n_e2e = max(4, args.steps)
+    n_e2e = max(8, args.steps)
     loaded = [torch.cuda.Event() for _ in range(2)]   # inputs of a set uploaded
     consumed = [torch.cuda.Event() for _ in range(2)]  # a set's step has run
 
@@ -457,7 +490,8 @@ def run_ours(args, rank, world, local_rank, raw):
         with torch.cuda.stream(copy_stream):
             if i >= 2:
                 copy_stream.wait_event(consumed[i % 2])
-            f_dev.copy_(feats_pin, non_blocking=True)
+            for sc in range(B):  # one copy a scene, as scenes arrive
+                f_dev[sc].copy_(feats_pin[sc], non_blocking=True)
             p_dev.copy_(pos_pin, non_blocking=True)
             t_dev.copy_(fr_pin, non_blocking=True)
             loaded[i % 2].record(copy_stream)
@@ -499,7 +533,8 @@ def run_ours(args, rank, world, local_rank, raw):
     e2e = {"value": B * world / (e2e_ms / 1000.0), "unit": "scenes/s",
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 3),
            "steps": n_e2e, "h2d_GBps": round(h2d_gbs, 1),
-           "overlap": "next step's upload on a copy stream during this step's selection"}
+           "overlap": "next step's upload (one copy a scene) on a copy stream during this "
+                      "step's selection"}
     del inputs
 
     if rank != 0:
