@@ -708,7 +708,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   hw_cluster_sync();  // every block initialised before any peer writes to it
 
   if (a.g0) {
-    // step 0 from the cost epilogue's partial row sums: the same terms as
+    // step 0 from the cost pass's partial row sums: the same terms as
     // the gain (exact products v d, each fused into a rounded sum), summed
     // in another order, so like the gain within gamma_(n-1) =
     // (n-1)u / (1 - (n-1)u) of the exact sum (u = 2^-24, n <= 16384 terms:
