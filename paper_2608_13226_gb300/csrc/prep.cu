@@ -604,45 +604,160 @@ __global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos,
     if (i >= KK - kk) out[i - (KK - kk)] = (int32_t)(best[i] & 0xFFFFFFFFull);
 }
 
-// The largest pinned-fp32 squared distance over pairs, into stats.d2_max_bits:
-// block of 256 rows, candidate tiles of 1024 in shared memory, only tiles
-// that reach past the block's first row (d^2 is symmetric).
-__global__ void __launch_bounds__(256) k_diameter_pairs(const float* __restrict__ pos, int N,
-                                                        SceneStats* stats) {
-  __shared__ float4 s_p[1024];
-  __shared__ uint32_t s_m[8];
-  const int b = blockIdx.y;
-  const int row0 = blockIdx.x * 256;
-  const float* X = pos + (size_t)b * N * 3;
-  const int i = row0 + threadIdx.x;
-  float qx = 0.f, qy = 0.f, qz = 0.f;
-  if (i < N) {
-    qx = X[3 * i];
-    qy = X[3 * i + 1];
-    qz = X[3 * i + 2];
+// The largest pinned-fp32 squared distance over pairs, into stats.d2_max_bits,
+// from the neighbour grid (points sorted by cell).  A lower bound L is the
+// largest d^2 among the extreme points of 13 directions (an actual pair).
+// For two cells whose coordinates differ by (dx, dy, dz) cells, any two of
+// their points are at most (|d| + 1) h + delta apart along each axis (delta
+// covers the rounding of the cell assignment), so the pair of cells can hold
+// a pair above L only if sum ((|d| + 1) h + delta)^2, inflated for fp32
+// rounding, reaches L.  Cells that reach L with no cell of the grid's corners
+// are dropped; the pairs of the remaining cells that pass the test are
+// evaluated with the same arithmetic as every other kernel, so the result is
+// exactly the largest d^2.  Blocks (part, scene); part p takes every P-th
+// row of candidate-cell pairs.
+constexpr int DIA_THREADS = 512, DIA_PARTS = 4, DIA_DIRS = 13;
+
+__device__ __forceinline__ uint32_t warp_max_u32(uint32_t v) {
+  for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float dia_dir_dot(int d, float x, float y, float z) {
+  switch (d) {
+    case 0: return x;
+    case 1: return y;
+    case 2: return z;
+    case 3: return x + y;
+    case 4: return x - y;
+    case 5: return x + z;
+    case 6: return x - z;
+    case 7: return y + z;
+    case 8: return y - z;
+    case 9: return x + y + z;
+    case 10: return x + y - z;
+    case 11: return x - y + z;
+    default: return -x + y + z;
   }
-  uint32_t dmax = 0u;
-  for (int base = (row0 / 1024) * 1024; base < N; base += 1024) {
-    const int n = min(1024, N - base);
+}
+
+__global__ void __launch_bounds__(DIA_THREADS) k_diameter_grid(
+    int N, int gmax, const GridInfo* __restrict__ info, const int32_t* __restrict__ cell_start,
+    const float4* __restrict__ sorted, SceneStats* stats) {
+  extern __shared__ int s_cand[];  // candidate cells, [gmax]
+  __shared__ unsigned long long s_ext[2 * DIA_DIRS];
+  __shared__ int s_ncand, s_wcnt[DIA_THREADS / 32];
+  __shared__ uint32_t s_m[DIA_THREADS / 32];
+  const int b = blockIdx.y;
+  const GridInfo g = info[b];
+  const int32_t* cs = cell_start + (size_t)b * (gmax + 1);
+  const float4* P = sorted + (size_t)b * N;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (threadIdx.x < 2 * DIA_DIRS) s_ext[threadIdx.x] = 0ull;
+  if (threadIdx.x == 0) s_ncand = 0;
+  __syncthreads();
+
+  // extreme points of 13 directions (max of +u and of -u), as (key, slot)
+  for (int d = 0; d < DIA_DIRS; ++d) {
+    unsigned long long hi = 0ull, lo = 0ull;
+    for (int i = threadIdx.x; i < N; i += DIA_THREADS) {
+      const float4 p = P[i];
+      const float v = dia_dir_dot(d, p.x, p.y, p.z);
+      const unsigned long long kh = ((unsigned long long)f2key(v) << 32) | (uint32_t)i;
+      const unsigned long long kl = ((unsigned long long)f2key(-v) << 32) | (uint32_t)i;
+      hi = kh > hi ? kh : hi;
+      lo = kl > lo ? kl : lo;
+    }
+    hi = warp_max_u64(hi);
+    lo = warp_max_u64(lo);
+    if (lane == 0) {
+      atomicMax(&s_ext[2 * d], hi);
+      atomicMax(&s_ext[2 * d + 1], lo);
+    }
+  }
+  __syncthreads();
+  uint32_t m = 0u;  // the largest d^2 bits this thread has seen
+  for (int e = threadIdx.x; e < 2 * DIA_DIRS * 2 * DIA_DIRS; e += DIA_THREADS) {
+    const int u = e / (2 * DIA_DIRS), v = e % (2 * DIA_DIRS);
+    const float4 a = P[(uint32_t)(s_ext[u] & 0xFFFFFFFFull)];
+    const float4 c = P[(uint32_t)(s_ext[v] & 0xFFFFFFFFull)];
+    m = max(m, __float_as_uint(sqdist_rn(a.x, a.y, a.z, c.x, c.y, c.z)));
+  }
+  m = warp_max_u32(m);
+  if (lane == 0) s_m[w] = m;
+  __syncthreads();
+  uint32_t Lb = s_m[0];
+  for (int i = 1; i < DIA_THREADS / 32; ++i) Lb = max(Lb, s_m[i]);
+  const float L = __uint_as_float(Lb);
+
+  // bound of two cells' d^2 from their coordinate differences
+  float span = 0.0f;
+  for (int a = 0; a < 3; ++a) span = fmaxf(span, fabsf(g.lo[a]) + (float)g.dims[a] * g.h);
+  const float delta = 1e-3f * g.h + 1e-5f * span;
+  auto bound = [&](int ax, int ay, int az, int bx, int by, int bz) -> float {
+    const float ex = (float)(abs(ax - bx) + 1) * g.h + delta;
+    const float ey = (float)(abs(ay - by) + 1) * g.h + delta;
+    const float ez = (float)(abs(az - bz) + 1) * g.h + delta;
+    return (ex * ex + ey * ey + ez * ez) * 1.000244140625f;  // 1 + 2^-12
+  };
+  // the candidate cells in ascending order (every block of the scene lists
+  // them alike, so the parts split the pairs without gaps or overlaps)
+  const int d0 = g.dims[0], d1 = g.dims[1], d2 = g.dims[2];
+  for (int base = 0; base < g.ncells; base += DIA_THREADS) {
+    const int c = base + threadIdx.x;
+    bool cand = false;
+    if (c < g.ncells && cs[c + 1] > cs[c]) {
+      const int cx = c % d0, cy = (c / d0) % d1, cz = c / (d0 * d1);
+      float far = 0.0f;
+      for (int k = 0; k < 8; ++k)
+        far = fmaxf(far, bound(cx, cy, cz, (k & 1) ? d0 - 1 : 0, (k & 2) ? d1 - 1 : 0,
+                               (k & 4) ? d2 - 1 : 0));
+      cand = far >= L;
+    }
+    const uint32_t bal = __ballot_sync(0xFFFFFFFFu, cand);
+    if (lane == 0) s_wcnt[w] = __popc(bal);
     __syncthreads();
-    for (int t = threadIdx.x; t < n; t += 256) {
-      const int k = base + t;
-      s_p[t] = make_float4(X[3 * k], X[3 * k + 1], X[3 * k + 2], 0.f);
+    int off = s_ncand;
+    for (int i = 0; i < w; ++i) off += s_wcnt[i];
+    if (cand) s_cand[off + __popc(bal & ((1u << lane) - 1u))] = c;
+    __syncthreads();  // every thread has read s_ncand and s_wcnt
+    if (threadIdx.x == 0) {
+      int tot = 0;
+      for (int i = 0; i < DIA_THREADS / 32; ++i) tot += s_wcnt[i];
+      s_ncand += tot;
     }
     __syncthreads();
-    if (i < N)
-      for (int t = 0; t < n; ++t) {
-        const float4 p = s_p[t];
-        dmax = max(dmax, __float_as_uint(sqdist_rn(qx, qy, qz, p.x, p.y, p.z)));
-      }
   }
-  for (int o = 16; o > 0; o >>= 1) dmax = max(dmax, __shfl_xor_sync(0xFFFFFFFFu, dmax, o));
-  if ((threadIdx.x & 31) == 0) s_m[threadIdx.x >> 5] = dmax;
+  const int M = s_ncand;
+
+  // rows of candidate-cell pairs: warp (part, w) takes rows r = part + P*w, ...
+  const int nw = DIA_THREADS / 32;
+  for (int r = blockIdx.x + DIA_PARTS * w; r < M; r += DIA_PARTS * nw) {
+    const int A = s_cand[r];
+    const int ax = A % d0, ay = (A / d0) % d1, az = A / (d0 * d1);
+    const int a0 = cs[A], a1 = cs[A + 1];
+    for (int t = r + lane; t < M; t += 32) {
+      const int Bc = s_cand[t];
+      const int bx = Bc % d0, by = (Bc / d0) % d1, bz = Bc / (d0 * d1);
+      if (bound(ax, ay, az, bx, by, bz) < L) continue;
+      const int b0 = cs[Bc], b1 = cs[Bc + 1];
+      for (int i = a0; i < a1; ++i) {
+        const float4 p = P[i];
+        for (int j = b0; j < b1; ++j) {
+          const float4 q = P[j];
+          m = max(m, __float_as_uint(sqdist_rn(p.x, p.y, p.z, q.x, q.y, q.z)));
+        }
+      }
+    }
+  }
+  m = warp_max_u32(m);
+  __syncthreads();  // every warp has read s_m above
+  if (lane == 0) s_m[w] = m;
   __syncthreads();
   if (threadIdx.x == 0) {
-    uint32_t m = s_m[0];
-    for (int w = 1; w < 8; ++w) m = max(m, s_m[w]);
-    atomicMax(&stats[b].d2_max_bits, m);
+    uint32_t mm = s_m[0];
+    for (int i = 1; i < nw; ++i) mm = max(mm, s_m[i]);
+    atomicMax(&stats[b].d2_max_bits, mm);
   }
 }
 
@@ -656,21 +771,23 @@ int launch_knn_grid(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr
                     SceneStats* stats, GridInfo* info, int32_t* cell_start, float4* sorted,
                     cudaStream_t s) {
   const int gmax = grid_cells_max(N);
-  {
-    dim3 grid((unsigned)((N + 255) / 256), (unsigned)B);
-    k_diameter_pairs<<<grid, 256, 0, s>>>(pos, (int)N, stats);
-    CP_TRY_STATUS(last_launch_status());
-  }
-  if (kk <= 0) return CP_OK;
   if (kk > 8) return CP_EINVAL;
   const size_t smem = sizeof(int) * (size_t)(gmax + 1);
   if (smem > 48 * 1024 &&
-      cuda_status(cudaFuncSetAttribute(k_grid_build, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem),
-                  "launch_knn_grid: smem attribute") != CP_OK)
+      (cuda_status(cudaFuncSetAttribute(k_grid_build, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)smem),
+                   "launch_knn_grid: smem attribute") != CP_OK ||
+       cuda_status(cudaFuncSetAttribute(k_diameter_grid,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                   "launch_knn_grid: smem attribute") != CP_OK))
     return CP_ECUDA;
   k_grid_build<<<(unsigned)B, 1024, smem, s>>>(pos, (int)N, gmax, info, cell_start, sorted);
   CP_TRY_STATUS(last_launch_status());
+  k_diameter_grid<<<dim3(DIA_PARTS, (unsigned)B), DIA_THREADS, smem, s>>>((int)N, gmax, info,
+                                                                          cell_start, sorted,
+                                                                          stats);
+  CP_TRY_STATUS(last_launch_status());
+  if (kk <= 0) return CP_OK;
   dim3 grid((unsigned)((N + 127) / 128), (unsigned)B);
   k_knn_grid<8><<<grid, 128, 0, s>>>(pos, (int)N, kk, gmax, info, cell_start, sorted, nbr);
   return last_launch_status();

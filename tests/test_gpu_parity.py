@@ -54,6 +54,57 @@ def test_knn_ties_and_duplicates(orc):
     np.testing.assert_array_equal(host(nbr), orc.knn_others(X, 11))
 
 
+def _max_d2_fp32(X):
+    """The largest squared distance over all pairs, every operation rounded
+    in fp32 in the kernels' order ((dx dx + dy dy) + dz dz)."""
+    X = np.asarray(X, np.float32)
+    best = np.float32(0.0)
+    for i0 in range(0, len(X), 512):
+        d = X[i0:i0 + 512, None, :] - X[None, :, :]
+        sq = d * d
+        best = max(best, ((sq[..., 0] + sq[..., 1]) + sq[..., 2]).max())
+    return best
+
+
+def _shapes(rng):
+    box = rng.random((3000, 3)).astype(np.float32) * np.float32([8, 6, 3])
+    th, ph = rng.random(2500) * 2 * np.pi, np.arccos(rng.uniform(-1, 1, 2500))
+    shell = np.stack([np.sin(ph) * np.cos(th), np.sin(ph) * np.sin(th), np.cos(ph)], 1)
+    line = np.zeros((700, 3), np.float32)
+    line[:, 0] = rng.random(700)
+    dup = np.repeat(rng.random((60, 3)).astype(np.float32), 5, axis=0)
+    return {"box": box, "walls": scene("long_video", 3, N=2048, D=16)["pos"],
+            "shell": (2.5 * shell).astype(np.float32), "line": line, "dup": dup,
+            "offset": box[:900] + np.float32(1000.0), "one": box[:1], "two": box[:2],
+            "same": np.repeat(box[:1], 33, axis=0)}
+
+
+@pytest.mark.parametrize("k", [8, 0])
+def test_diameter_from_grid_is_exact(k):
+    # the grid path (k <= 8) prunes cell pairs by a bound: its diameter must
+    # be exactly the largest pinned-fp32 d^2 over all pairs, whatever the shape
+    rng = np.random.default_rng(21)
+    for name, X in _shapes(rng).items():
+        pos = torch.from_numpy(np.ascontiguousarray(X, np.float32)).cuda()
+        _, dia = cp.coverprune_knn(pos, min(k, len(X) - 1))
+        got = float(host(dia))
+        want = float(np.sqrt(np.float32(_max_d2_fp32(X)), dtype=np.float32))
+        assert got == want, f"{name}: {got} != {want}"
+
+
+def test_diameter_grid_equals_brute_force_batched():
+    rng = np.random.default_rng(22)
+    X = (rng.random((3, 1500, 3)) * np.float32([8, 8, 3])).astype(np.float32)
+    X[1, :, 2] = 0.0  # a flat scene
+    pos = torch.from_numpy(X).cuda()
+    _, dia = cp.coverprune_knn(pos, 8)
+    nbr = torch.empty(3, 1500, 8, dtype=torch.int32, device="cuda")
+    dia_bf = torch.empty(3, dtype=torch.float32, device="cuda")
+    cp.coverprune_knn_noalloc(pos, nbr, dia_bf)
+    torch.cuda.synchronize()
+    assert torch.equal(dia, dia_bf)
+
+
 # --------------------------------------------------------------------------
 # K0-K4: normalisers, cost, capacity
 # --------------------------------------------------------------------------
