@@ -37,6 +37,7 @@ METRIC = "scenes/sec & pruning latency (N=8192,D=3584,15% keep); % HBM / tensor 
 WORKLOAD = "batch32_long_video_full_sgs_15pct"
 SCENES, RETENTION = 32, 0.15
 SCENE_NAME = "long_video"
+LOCAL_G = 64  # local neighbourhood size of the local-SGS measurement
 STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output")
 
 
@@ -436,6 +437,37 @@ def run_ours(args, rank, world, local_rank, raw):
     latency_ms = statistics.median(lat)
     del ws1
 
+    # local SGS (Eq. local_neighbor with g = 64) on the same batch
+    prm_loc = cp.Params(g=LOCAL_G)
+    wsg = cp.workspace(cp.CP_OP_SELECT, B, N, D, K, cp.CP_BF16, prm_loc, dev)
+    for _ in range(args.warmup):
+        cp.coverprune_select(feats, pos, fr, K, prm_loc, order=False, gains=False, ws=wsg,
+                             out=out)
+    barrier()
+    cp.coverprune_profile_read()
+    cp.coverprune_profile_enable(True)
+    a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        cp.coverprune_select(feats, pos, fr, K, prm_loc, order=False, gains=False, ws=wsg,
+                             out=out)
+    b_.record(stream)
+    barrier()
+    cp.coverprune_profile_enable(False)
+    gprof = cp.coverprune_profile_read()
+    gstats = cp.coverprune_call_stats(wsg)
+    st = cp.coverprune_check(wsg)
+    if st != cp.CP_OK:
+        raise RuntimeError(f"device status after the local-SGS steps: {cp.status_string(st)}")
+    loc_ms = max_over_ranks(a.elapsed_time(b_) / args.steps)
+    loc_sgs_ms = gprof["sgs"][0] / args.steps if gprof["sgs"][0] > 0 else None
+    local = {"g": LOCAL_G, "scenes_per_s": B * world / (loc_ms / 1000.0),
+             "ms_per_step": round(loc_ms, 3),
+             "sgs_us_per_greedy_step": loc_sgs_ms and round(1000.0 * loc_sgs_ms / K, 3),
+             "gain_evaluations_per_step": gstats["gain_evaluations"],
+             "stages_ms": {k: round(v[0] / args.steps, 3) for k, v in gprof.items() if v[0] > 0}}
+    del wsg
+
     # CoverPrune-Lite on the same batch
     wsl = cp.workspace(cp.CP_OP_LITE, B, N, D, K, cp.CP_BF16, prm, dev)
     lite_out = {"kept": torch.empty(B, K, dtype=torch.int64, device=dev)}
@@ -557,7 +589,7 @@ def run_ours(args, rank, world, local_rank, raw):
                        "generator": "paper_2608_13226_gb300.scenes long_video, seeds "
                                     f"{rank * B}..{rank * B + B - 1} per rank"},
             "latency_ms": round(latency_ms, 3),
-            "lite": lite, "roofline": roofline, "roofline_sgs": roofline_sgs,
+            "lite": lite, "local_sgs": local, "roofline": roofline, "roofline_sgs": roofline_sgs,
             "roofline_front": roofline_front, "sgs_full_sweep": sweep,
             "stages_ms": stages, "gpu_launches": gpu_launches, "e2e": e2e,
             "clocks": clocks, "cpu_baseline": cpu}

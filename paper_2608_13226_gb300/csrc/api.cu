@@ -193,7 +193,7 @@ static DevParams dev_params(const cp_params* p, int64_t N) {
 // ---------------------------------------------------------------------------
 struct Plan {
   size_t hdr, counters, stats, norms, inv, tok, nbr, r, v;
-  size_t grid_info, grid_start, grid_pts;         // neighbour grid (kk <= 8)
+  size_t grid_info, grid_start, grid_pts;         // neighbour grid (kk <= kKnnGridMax)
   size_t cost, slab, partials, order32, g0;       // select
   size_t perm, prefix, gs, proto, score;          // lite
   size_t total;
@@ -228,7 +228,7 @@ static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d,
   pl->inv = take(sizeof(float) * BN);
   pl->tok = take(sizeof(float4) * BN);
   pl->nbr = take(sizeof(int32_t) * BN * (size_t)d.kk);
-  if (d.kk <= 8) {
+  if (d.kk <= kKnnGridMax) {
     pl->grid_info = take(sizeof(GridInfo) * (size_t)B);
     pl->grid_start = take(sizeof(int32_t) * (size_t)B * (size_t)(grid_cells_max(N) + 1));
     pl->grid_pts = take(sizeof(float4) * BN);
@@ -291,7 +291,7 @@ static int run_front(const void* feats, int dtype, const float* pos, const int32
     CP_TRY(launch_scene_stats(pos, frame, B, N, stats, s));
     CP_TRY(launch_inv_norms(feats, dtype, pos, B, N, D, at<float>(ws, pl.inv),
                             at<float4>(ws, pl.tok), s));
-    if (d.kk <= 8)
+    if (d.kk <= kKnnGridMax)
       CP_TRY(launch_knn_grid(pos, B, N, d.kk, at<int32_t>(ws, pl.nbr), stats,
                              at<GridInfo>(ws, pl.grid_info), at<int32_t>(ws, pl.grid_start),
                              at<float4>(ws, pl.grid_pts), s));
@@ -482,9 +482,15 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
   }
   // the dense lazy selection starts from bounds the cost pass sums
   float* g0 = (dtype == CP_BF16 && d.g >= N && d.sgs_mode == 0) ? at<float>(ws, pl.g0) : nullptr;
+  // local SGS reads only the N x g slab: for bf16 it comes straight from
+  // the stored cosines, and the dense cost is never formed
+  float* slab = d.g < N ? at<float>(ws, pl.slab) : nullptr;
   {
     Stage st(CP_STAGE_COST, s);
-    if (dtype == CP_BF16)
+    if (dtype == CP_BF16 && slab)
+      CP_TRY(launch_slab_cos(C, pl.ldc, nbr, at<float4>(ws, pl.tok), frame, nm, d, B, N, slab,
+                             s));
+    else if (dtype == CP_BF16)
       CP_TRY(launch_fst_apply(C, pl.ldc, B, N, at<float4>(ws, pl.tok), frame, nm, d, v, g0, s));
     else
       CP_TRY(launch_cost(feats, dtype, inv, at<float4>(ws, pl.tok), pos, frame, nm, d, B, N, D, C,
@@ -493,11 +499,7 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
   int32_t* order32 = at<int32_t>(ws, pl.order32);
   {
     Stage st(CP_STAGE_SGS, s);
-    float* slab = nullptr;
-    if (d.g < N) {
-      slab = at<float>(ws, pl.slab);
-      CP_TRY(launch_slab(C, pl.ldc, nbr, d, B, N, slab, s));
-    }
+    if (slab && dtype != CP_BF16) CP_TRY(launch_slab(C, pl.ldc, nbr, d, B, N, slab, s));
     CP_TRY(launch_sgs(C, pl.ldc, slab, nbr, v, d, B, N, K, order32, gains, objective,
                       at<uint64_t>(ws, pl.partials), at<uint32_t>(ws, pl.counters), status, s,
                       g0));
@@ -572,7 +574,7 @@ int coverprune_knn(const float* pos, int64_t B, int64_t N, int64_t k, int32_t* n
   SceneStats* stats = at<SceneStats>(ws, st_off);
   CP_TRY(cuda_status(cudaMemsetAsync(ws, 0, sizeof(int), s)));
   CP_TRY(launch_scene_stats(pos, nullptr, B, N, stats, s));  // frames are not needed
-  if (k <= 8)
+  if (k <= kKnnGridMax)
     CP_TRY(launch_knn_grid(pos, B, N, (int)k, k > 0 ? nbr : nullptr, stats,
                            at<GridInfo>(ws, gi_off), at<int32_t>(ws, gs_off),
                            at<float4>(ws, gp_off), s));

@@ -812,7 +812,39 @@ __global__ void __launch_bounds__(256, 3)
   }
 }
 
+// The local neighbourhoods' costs straight from the stored cosines:
+// slab[b][t][k] = C(t, M_g(t)[k]) with M_g(t)[0] = t and M_g(t)[k] the k-th
+// nearest other token, by the same arithmetic as k_fst_apply (the slab holds
+// exactly the entries the dense cost would).  One thread per (t, k).
+__global__ void __launch_bounds__(256) k_slab_cos(const float* __restrict__ cos, int64_t ldc, int N,
+                                                  int g, int kk, const int32_t* __restrict__ nbr,
+                                                  const float4* __restrict__ tok,
+                                                  const int32_t* __restrict__ frame,
+                                                  const SceneNorms* __restrict__ norms,
+                                                  DevParams P, float* __restrict__ slab) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int b = blockIdx.y;
+  if (i >= (int64_t)N * g) return;
+  const int t = (int)(i / g), k = (int)(i % g);
+  const size_t sb = (size_t)b * N;
+  const int j = k == 0 ? t : __ldg(nbr + (sb + t) * kk + (k - 1));
+  const FstConst kf = fst_const(norms[b], P);
+  const float4 ti = __ldg(tok + sb + t), tj = __ldg(tok + sb + j);
+  const float c = __ldg(cos + (sb + t) * (size_t)ldc + j);
+  slab[sb * g + i] = fst_cost_fold(kf, c, ti.x - tj.x, ti.y - tj.y, ti.z - tj.z,
+                                   (float)__ldg(frame + sb + t), (float)__ldg(frame + sb + j));
+}
+
 }  // namespace
+
+int launch_slab_cos(const float* cos, int64_t ldc, const int32_t* nbr, const float4* tok,
+                    const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
+                    int64_t N, float* slab, cudaStream_t s) {
+  const int64_t n = N * P.g;
+  dim3 grid((unsigned)((n + 255) / 256), (unsigned)B);
+  k_slab_cos<<<grid, 256, 0, s>>>(cos, ldc, (int)N, P.g, P.kk, nbr, tok, frame, norms, P, slab);
+  return last_launch_status();
+}
 
 int fst_apply_slots(int64_t ldc) { return (int)((ldc + FA_COLS - 1) / FA_COLS); }
 

@@ -100,6 +100,8 @@ int launch_inv_norms(const void* feats, int dtype, const float* pos, int64_t B, 
 // K1: per token the kk nearest other tokens by (fp32 d^2, index) into
 // nbr[(b*N + j)*kk + q]; also the scene's largest squared distance.
 int grid_cells_max(int64_t N);
+// Neighbour counts the grid search serves (larger ones take the brute-force kernels).
+constexpr int kKnnGridMax = 128;
 int launch_knn_grid(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr,
                     SceneStats* stats, GridInfo* info, int32_t* cell_start, float4* sorted,
                     cudaStream_t s);
@@ -131,6 +133,11 @@ int launch_capacity(const void* feats, int dtype, const float* inv, const float*
                     const DevParams& P, int64_t B, int64_t N, int64_t D, float* r, float* v,
                     float* v_out, cudaStream_t s, const float* cos = nullptr,
                     int64_t ldc = 0);
+// Local SGS, bf16 features: the same slab computed from the stored cosines
+// (cos [B][N][ldc], as the normaliser pass writes them), without a dense cost.
+int launch_slab_cos(const float* cos, int64_t ldc, const int32_t* nbr, const float4* tok,
+                    const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
+                    int64_t N, float* slab, cudaStream_t s);
 // Local SGS: slab[b][t][k] = C(t, M_g(t)[k]) gathered from the dense cost.
 int launch_slab(const float* cost, int64_t ldc, const int32_t* nbr, const DevParams& P,
                 int64_t B, int64_t N, float* slab, cudaStream_t s);

@@ -424,7 +424,7 @@ int launch_knn(const float* pos, const float4* tok, int64_t B, int64_t N, int kk
 }
 
 // ---------------------------------------------------------------------------
-// K1 through a uniform grid (kk <= 8): exact, with the same keys and lists
+// K1 through a uniform grid (kk <= kKnnGridMax): exact, with the same keys and lists
 // as the brute-force kernels, but each query visits only the cells around
 // it.  The scene's bounding box is cut into cubic cells of side h =
 // (largest extent) / G with G = the least integer such that 4 G^3 >= N, so
@@ -604,6 +604,107 @@ __global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos,
     if (i >= KK - kk) out[i - (KK - kk)] = (int32_t)(best[i] & 0xFFFFFFFFull);
 }
 
+// More neighbours (8 < kk <= kKnnGridMax): the same shell search, one thread
+// per query, with the kk best keys in a max-heap in shared memory (slot i of
+// thread t at [i][t]: the threads of a warp touch distinct banks); the root
+// is the worst kept key.  A heapsort leaves them ascending at the end.
+__global__ void __launch_bounds__(128) k_knn_grid_heap(const float* __restrict__ pos, int N, int kk,
+                                                       int gmax, const GridInfo* __restrict__ info,
+                                                       const int32_t* __restrict__ cell_start,
+                                                       const float4* __restrict__ sorted,
+                                                       int32_t* __restrict__ nbr) {
+  extern __shared__ unsigned long long s_heap[];  // [kk][blockDim.x]
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  const int b = blockIdx.y;
+  if (j >= N) return;
+  const int T = blockDim.x;
+  unsigned long long* H = s_heap + threadIdx.x;  // H[i * T] is slot i
+  const GridInfo g = info[b];
+  const float* X = pos + (size_t)b * N * 3;
+  const int32_t* cs = cell_start + (size_t)b * (gmax + 1);
+  const float4* P = sorted + (size_t)b * N;
+  const float qx = X[3 * j], qy = X[3 * j + 1], qz = X[3 * j + 2];
+  const int cx = grid_coord(g, qx, 0), cy = grid_coord(g, qy, 1), cz = grid_coord(g, qz, 2);
+  int cnt = 0;
+  unsigned long long worst = ~0ull;  // the root once the heap is full
+  // the root replaced by key (smaller than it), sifted down within n slots
+  auto sift_down = [&](unsigned long long key, int n) {
+    int i = 0;
+    for (;;) {
+      const int l = 2 * i + 1;
+      if (l >= n) break;
+      const int r = l + 1;
+      unsigned long long ck = H[(size_t)l * T];
+      int c = l;
+      if (r < n) {
+        const unsigned long long rk = H[(size_t)r * T];
+        if (rk > ck) {
+          ck = rk;
+          c = r;
+        }
+      }
+      if (ck <= key) break;
+      H[(size_t)i * T] = ck;
+      i = c;
+    }
+    H[(size_t)i * T] = key;
+  };
+  const int rmax = max(g.dims[0], max(g.dims[1], g.dims[2]));
+  for (int r = 0; r <= rmax; ++r) {
+    for (int dz = -r; dz <= r; ++dz) {
+      const int z = cz + dz;
+      if (z < 0 || z >= g.dims[2]) continue;
+      for (int dy = -r; dy <= r; ++dy) {
+        const int y = cy + dy;
+        if (y < 0 || y >= g.dims[1]) continue;
+        const bool face = dz == -r || dz == r || dy == -r || dy == r;
+        for (int dx = -r; dx <= r; dx += (face || r == 0) ? 1 : 2 * r) {
+          const int x = cx + dx;
+          if (x < 0 || x >= g.dims[0]) continue;
+          const int c = (z * g.dims[1] + y) * g.dims[0] + x;
+          const int e = cs[c + 1];
+          for (int s = cs[c]; s < e; ++s) {
+            const float4 p = P[s];
+            const int k = __float_as_int(p.w);
+            const uint32_t bits = __float_as_uint(sqdist_rn(qx, qy, qz, p.x, p.y, p.z));
+            if (k == j || bits > (uint32_t)(worst >> 32)) continue;
+            const unsigned long long key = ((unsigned long long)bits << 32) | (uint32_t)k;
+            if (key >= worst) continue;
+            if (cnt < kk) {  // filling: sift the new key up
+              int i = cnt++;
+              while (i > 0) {
+                const int pi = (i - 1) >> 1;
+                const unsigned long long pk = H[(size_t)pi * T];
+                if (pk >= key) break;
+                H[(size_t)i * T] = pk;
+                i = pi;
+              }
+              H[(size_t)i * T] = key;
+              if (cnt == kk) worst = H[0];
+            } else {
+              sift_down(key, kk);
+              worst = H[0];
+            }
+          }
+        }
+      }
+    }
+    if (cnt == kk) {  // the heap is full: is anything closer still possible?
+      const float reach = ((float)r - 1.0f / 1024.0f) * g.h;
+      if (reach > 0.0f && __uint_as_float((uint32_t)(worst >> 32)) < reach * reach) break;
+    }
+  }
+  // heapsort: the largest to the end, repeatedly
+  for (int n = kk; n > 1; --n) {
+    const unsigned long long top = H[0];
+    const unsigned long long last = H[(size_t)(n - 1) * T];
+    H[(size_t)(n - 1) * T] = top;
+    sift_down(last, n - 1);
+  }
+  int32_t* out = nbr + ((size_t)b * N + j) * kk;
+  for (int i = 0; i < kk; ++i) out[i] = (int32_t)(H[(size_t)i * T] & 0xFFFFFFFFull);
+}
+
 // The largest pinned-fp32 squared distance over pairs, into stats.d2_max_bits,
 // from the neighbour grid (points sorted by cell).  A lower bound L is the
 // largest d^2 among the extreme points of 13 directions (an actual pair).
@@ -771,7 +872,7 @@ int launch_knn_grid(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr
                     SceneStats* stats, GridInfo* info, int32_t* cell_start, float4* sorted,
                     cudaStream_t s) {
   const int gmax = grid_cells_max(N);
-  if (kk > 8) return CP_EINVAL;
+  if (kk > kKnnGridMax) return CP_EINVAL;
   const size_t smem = sizeof(int) * (size_t)(gmax + 1);
   if (smem > 48 * 1024 &&
       (cuda_status(cudaFuncSetAttribute(k_grid_build, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -788,8 +889,20 @@ int launch_knn_grid(const float* pos, int64_t B, int64_t N, int kk, int32_t* nbr
                                                                           stats);
   CP_TRY_STATUS(last_launch_status());
   if (kk <= 0) return CP_OK;
-  dim3 grid((unsigned)((N + 127) / 128), (unsigned)B);
-  k_knn_grid<8><<<grid, 128, 0, s>>>(pos, (int)N, kk, gmax, info, cell_start, sorted, nbr);
+  if (kk <= 8) {
+    dim3 grid((unsigned)((N + 127) / 128), (unsigned)B);
+    k_knn_grid<8><<<grid, 128, 0, s>>>(pos, (int)N, kk, gmax, info, cell_start, sorted, nbr);
+    return last_launch_status();
+  }
+  const int T = kk <= 64 ? 128 : 64;  // heaps of T x kk keys: at most 64 KB
+  const size_t hsmem = sizeof(unsigned long long) * (size_t)T * (size_t)kk;
+  if (hsmem > 48 * 1024 &&
+      cuda_status(cudaFuncSetAttribute(k_knn_grid_heap, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)hsmem),
+                  "launch_knn_grid: heap smem attribute") != CP_OK)
+    return CP_ECUDA;
+  dim3 grid((unsigned)((N + T - 1) / T), (unsigned)B);
+  k_knn_grid_heap<<<grid, T, hsmem, s>>>(pos, (int)N, kk, gmax, info, cell_start, sorted, nbr);
   return last_launch_status();
 }
 
