@@ -195,6 +195,7 @@ struct Plan {
   size_t hdr, counters, stats, norms, inv, tok, nbr, r, v;
   size_t grid_info, grid_start, grid_pts;         // neighbour grid (kk <= kKnnGridMax)
   size_t cost, slab, partials, order32, g0;       // select
+  size_t rev_off, rev;                            // local SGS reverse neighbourhoods
   size_t perm, prefix, gs, proto, score;          // lite
   size_t total;
   int64_t ldc;
@@ -237,7 +238,11 @@ static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d,
   pl->v = take(sizeof(float) * BN);
   if (op == CP_OP_SELECT) {
     pl->cost = take(sizeof(float) * BN * (size_t)pl->ldc);
-    if (d.g < N) pl->slab = take(sizeof(float) * BN * (size_t)d.g);
+    if (d.g < N) {
+      pl->slab = take(sizeof(float) * BN * (size_t)d.g);
+      pl->rev_off = take(sizeof(int32_t) * (BN + (size_t)B));
+      pl->rev = take(sizeof(int32_t) * BN * (size_t)d.g);
+    }
     pl->partials = take(sizeof(uint64_t) * (size_t)sgs_partials_count(B, N));
     pl->order32 = take(sizeof(int32_t) * (size_t)B * (size_t)K);
     pl->g0 = take(sizeof(float) * BN * (size_t)fst_apply_slots(pl->ldc));
@@ -502,7 +507,8 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
     if (slab && dtype != CP_BF16) CP_TRY(launch_slab(C, pl.ldc, nbr, d, B, N, slab, s));
     CP_TRY(launch_sgs(C, pl.ldc, slab, nbr, v, d, B, N, K, order32, gains, objective,
                       at<uint64_t>(ws, pl.partials), at<uint32_t>(ws, pl.counters), status, s,
-                      g0));
+                      g0, slab ? at<int32_t>(ws, pl.rev_off) : nullptr,
+                      slab ? at<int32_t>(ws, pl.rev) : nullptr));
   }
   Stage st(CP_STAGE_OUTPUT, s);
   CP_TRY(launch_sort_kept(order32, B, K, kept, order, s));

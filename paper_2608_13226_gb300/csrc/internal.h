@@ -144,11 +144,14 @@ int launch_slab(const float* cost, int64_t ldc, const int32_t* nbr, const DevPar
 // Column tiles of the elementwise cost pass: the number of partial row sums
 // it writes per row into g0, [B][fst_apply_slots(ldc)][N].
 int fst_apply_slots(int64_t ldc);
-// K5: K greedy steps; order32[b*K + l] = token added at step l.
+// K5: K greedy steps; order32[b*K + l] = token added at step l.  Local
+// lazy SGS (g < N) also needs rev_off [B][N+1] and rev [B][N*g] (scratch for
+// the reverse neighbourhoods).
 int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
                int32_t* order32, float* gains, double* objective, uint64_t* partials,
-               uint32_t* counters, int* status, cudaStream_t s, const float* g0 = nullptr);
+               uint32_t* counters, int* status, cudaStream_t s, const float* g0 = nullptr,
+               int32_t* rev_off = nullptr, int32_t* rev = nullptr);
 // Sort the B rows of K int32 indices ascending into int64 (and copy the
 // unsorted order out as int64 if order64 != NULL).
 int launch_sort_kept(const int32_t* idx32, int64_t B, int64_t K, int64_t* kept,

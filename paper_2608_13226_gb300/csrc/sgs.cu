@@ -387,92 +387,152 @@ static int sgs_launch_impl(const float* cost, int64_t ldc, const float* slab, co
 // (gain_term is monotone in m and m only decreases), so the step's winner --
 // the largest (gain, -index) key -- is found without evaluating every
 // candidate: keep the last computed gain ub[t] of every token; a candidate
-// whose bound is exact this step ("fresh") and larger than every other bound
-// is the winner.  One block of 32 warps per scene; warp w owns the
-// candidates [w*S, (w+1)*S).  Each round every warp reports the largest
-// bound of its slice; if the overall largest is fresh the step is decided,
-// otherwise each warp whose slice-best is stale and could still beat the
-// best fresh key recomputes that row.  Step 0 evaluates every candidate.
-// No inter-block synchronisation: blocks are independent scenes.
+// whose bound is exact ("fresh") and larger than every other bound is the
+// winner.
 // ---------------------------------------------------------------------------
 constexpr int LZ_THREADS = 1024;
 constexpr int LZ_WARPS = LZ_THREADS / 32;
 
-template <bool LOCAL>
-__global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
-    const float* __restrict__ cost, int64_t ldc, const float* __restrict__ slab,
-    const int32_t* __restrict__ nbr, const float* __restrict__ v_all, DevParams P, int N, int K,
+// Reverse neighbourhoods of the local SGS, per scene in CSR form:
+// rev[rev_off[j] .. rev_off[j+1]) = the t with j in M_g(t) (M_g(t)[0] = t,
+// M_g(t)[k] = nbr[t][k-1]), in no particular order.  One block per scene;
+// counts and cursors in shared memory [N].
+__global__ void __launch_bounds__(1024) k_rev_build(const int32_t* __restrict__ nbr_all, int N,
+                                                    int g, int kk, int32_t* __restrict__ off_all,
+                                                    int32_t* __restrict__ rev_all) {
+  extern __shared__ int s_c[];  // [N]
+  __shared__ int s_sum[1024];
+  const int b = blockIdx.x;
+  const int32_t* NB = nbr_all + (size_t)b * N * kk;
+  int32_t* off = off_all + (size_t)b * (N + 1);
+  int32_t* rev = rev_all + (size_t)b * N * g;
+  const int64_t ng = (int64_t)N * g;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) s_c[j] = 0;
+  __syncthreads();
+  for (int64_t i = threadIdx.x; i < ng; i += blockDim.x) {
+    const int t = (int)(i / g), k = (int)(i % g);
+    atomicAdd(&s_c[k == 0 ? t : NB[(size_t)t * kk + (k - 1)]], 1);
+  }
+  __syncthreads();
+  // exclusive prefix of the counts: each thread a contiguous chunk, then a
+  // scan of the 1024 chunk sums
+  const int chunk = (N + blockDim.x - 1) / blockDim.x;
+  const int c0 = min(N, (int)threadIdx.x * chunk), c1 = min(N, c0 + chunk);
+  int part = 0;
+  for (int j = c0; j < c1; ++j) part += s_c[j];
+  s_sum[threadIdx.x] = part;
+  __syncthreads();
+  for (int d = 1; d < (int)blockDim.x; d <<= 1) {
+    const int x = threadIdx.x >= (unsigned)d ? s_sum[threadIdx.x - d] : 0;
+    __syncthreads();
+    s_sum[threadIdx.x] += x;
+    __syncthreads();
+  }
+  int run = s_sum[threadIdx.x] - part;  // the exclusive prefix of this chunk
+  for (int j = c0; j < c1; ++j) {
+    const int n = s_c[j];
+    off[j] = run;
+    s_c[j] = run;  // from here on: the next free slot of j
+    run += n;
+  }
+  if (threadIdx.x == 0) off[N] = (int)ng;
+  __syncthreads();
+  for (int64_t i = threadIdx.x; i < ng; i += blockDim.x) {
+    const int t = (int)(i / g), k = (int)(i % g);
+    const int j = k == 0 ? t : NB[(size_t)t * kk + (k - 1)];
+    rev[atomicAdd(&s_c[j], 1)] = t;
+  }
+}
+
+// Local SGS (g < N, Eq. local_neighbor), lazy, one block of 32 warps per
+// scene; warp w owns the candidates t = w (mod 32), so the tokens near a pick
+// (nearby indices), whose bounds go stale together, are re-evaluated by
+// different warps in the same round.  The update of a pick w
+// lowers m only on M_g(w), so gain(t) changes only if M_g(t) holds a target
+// whose m dropped: exactly the t on that target's reverse list.  Those lose
+// their exact mark ("dirty set"); every other bound stays exact -- its terms,
+// and so its rounded sum, are unchanged.  A round reads every warp's best key
+// and whether it is exact: if the block's largest is exact it is the winner,
+// otherwise each warp whose best is stale and above the largest exact one
+// re-evaluates it (one warp a row, local_row_gain) and rescans its slice.
+// Step 0 evaluates every candidate; no inter-block synchronisation.
+__global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_local(
+    const float* __restrict__ slab, const int32_t* __restrict__ nbr,
+    const float* __restrict__ v_all, const int32_t* __restrict__ rev_off_all,
+    const int32_t* __restrict__ rev_all, DevParams P, int N, int K,
     int32_t* __restrict__ order32, float* __restrict__ gains, double* __restrict__ objective,
     int* status) {
   extern __shared__ __align__(16) unsigned char smem[];
-  const int ncols = LOCAL ? N : (int)ldc;
   const int nwords = (N + 31) >> 5;
-  float* sm_m = reinterpret_cast<float*>(smem);                 // [ncols] coverage cost
-  float* sm_v = sm_m + ncols;                                   // [ncols] capacity
-  float* ub = sm_v + ncols;                                     // [N] last computed gain
-  uint32_t* chosen = reinterpret_cast<uint32_t*>(ub + N);       // [nwords]
-  uint32_t* fresh = chosen + nwords;                            // [nwords]
-  __shared__ unsigned long long s_wkey[LZ_WARPS];
-  __shared__ int s_wfresh[LZ_WARPS];
-  unsigned long long my_evals = 0ull, my_rounds = 0ull;  // lane 0 / thread 0 count
-  unsigned long long my_update_bytes = 0ull;              // thread 0
+  float* sm_m = reinterpret_cast<float*>(smem);            // [N] coverage cost
+  float* sm_v = sm_m + N;                                  // [N] capacity
+  float* ub = sm_v + N;                                    // [N] last computed gain
+  uint32_t* chosen = reinterpret_cast<uint32_t*>(ub + N);  // [nwords]
+  uint32_t* fresh = chosen + nwords;                       // [nwords]
+  __shared__ unsigned long long s_wkey[LZ_WARPS];          // each warp's best key
+  __shared__ int s_wfr[LZ_WARPS];                          // ... and whether it is exact
+  __shared__ int s_pick, s_bad;
+  unsigned long long my_evals = 0ull, my_rounds = 0ull, my_bytes = 0ull;
 
   const int b = blockIdx.x;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = P.g, kk = P.kk;
   const float* v = v_all + (size_t)b * N;
-  const float* Cb = LOCAL ? nullptr : cost + (size_t)b * N * ldc;
-  const float* Sb = LOCAL ? slab + (size_t)b * N * P.g : nullptr;
-  const int32_t* NB = nbr + (size_t)b * N * P.kk;
+  const float* Sb = slab + (size_t)b * N * g;
+  const int32_t* NB = nbr + (size_t)b * N * kk;
+  const int32_t* roff = rev_off_all + (size_t)b * (N + 1);
+  const int32_t* rev = rev_all + (size_t)b * N * g;
 
-  for (int j = threadIdx.x; j < ncols; j += LZ_THREADS) {
-    sm_m[j] = j < N ? P.m0 : 0.0f;
-    sm_v[j] = j < N ? v[j] : 0.0f;
+  for (int j = threadIdx.x; j < N; j += LZ_THREADS) {
+    sm_m[j] = P.m0;
+    sm_v[j] = v[j];
   }
-  for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) chosen[i] = 0u;
+  for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) {
+    chosen[i] = 0u;
+    fresh[i] = ~0u;
+  }
   __syncthreads();
-
   auto gain_of = [&](int t) -> float {
-    return LOCAL ? local_row_gain(Sb + (size_t)t * P.g, NB + (size_t)t * P.kk, t, P.g, sm_m, sm_v,
-                                  lane)
-                 : dense_row_gain(Cb + (size_t)t * ldc, sm_m, sm_v, ncols, lane);
+    return local_row_gain(Sb + (size_t)t * g, NB + (size_t)t * kk, t, g, sm_m, sm_v, lane);
   };
-  // step 0: every gain exactly
-  for (int t = w; t < N; t += LZ_WARPS) {
+  for (int t = w; t < N; t += LZ_WARPS) {  // step 0: every gain exactly
     const float g0 = gain_of(t);
     if (lane == 0) ub[t] = g0;
     ++my_evals;
   }
-  const int S = (N + LZ_WARPS - 1) / LZ_WARPS;
-  const int t_lo = w * S, t_hi = min(N, t_lo + S);
+  __syncthreads();
+  auto is_fresh = [&](unsigned long long key) -> int {
+    const int t = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
+    return key != 0ull && ((fresh[t >> 5] >> (t & 31)) & 1u);
+  };
+  auto rescan = [&]() {
+    unsigned long long best = 0ull;
+    for (int t = w + LZ_WARPS * lane; t < N; t += LZ_WARPS * 32)
+      if (!(chosen[t >> 5] & (1u << (t & 31)))) {
+        const unsigned long long key = gain_key(ub[t], t);
+        best = key > best ? key : best;
+      }
+    best = warp_max_u64(best);
+    if (lane == 0) {
+      s_wkey[w] = best;
+      s_wfr[w] = is_fresh(best);
+    }
+  };
+  rescan();
+  __syncthreads();
 
   for (int step = 0; step < K; ++step) {
-    for (int i = threadIdx.x; i < nwords; i += LZ_THREADS) fresh[i] = step == 0 ? ~0u : 0u;
-    __syncthreads();
     int pick = -1;
     for (int round = 0; round <= N; ++round) {
       ++my_rounds;
-      unsigned long long best = 0ull;
-      for (int t = t_lo + lane; t < t_hi; t += 32)
-        if (!(chosen[t >> 5] & (1u << (t & 31)))) {
-          const unsigned long long key = gain_key(ub[t], t);
-          best = key > best ? key : best;
-        }
-      best = warp_max_u64(best);
-      if (lane == 0) {
-        const int bt = (int)(0xFFFFFFFFu - (uint32_t)(best & 0xFFFFFFFFull));
-        s_wkey[w] = best;
-        s_wfresh[w] = best != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
-      }
-      __syncthreads();
-      unsigned long long G = 0ull, BF = 0ull;
-      for (int i = 0; i < LZ_WARPS; ++i) {
-        const unsigned long long k = s_wkey[i];
-        G = k > G ? k : G;
-        if (s_wfresh[i]) BF = k > BF ? k : BF;
-      }
-      const unsigned long long mine = s_wkey[w];
-      const bool mine_fresh = s_wfresh[w] != 0;
-      __syncthreads();  // s_wkey / s_wfresh are rewritten next round
+      // lane i reads warp i's entry; two warp maxima give G and BF
+      const unsigned long long ki = s_wkey[lane];
+      const int fi = s_wfr[lane];
+      const unsigned long long G = warp_max_u64(ki);
+      const unsigned long long BF = warp_max_u64(fi ? ki : 0ull);
+      const unsigned long long mine = __shfl_sync(0xFFFFFFFFu, ki, w);
+      const bool mine_fresh = __shfl_sync(0xFFFFFFFFu, fi, w) != 0;
+      __syncthreads();  // every warp has read s_wkey / s_wfr before any rescan
       if (G != 0ull && G == BF) {  // the largest bound is exact: the winner
         pick = (int)(0xFFFFFFFFu - (uint32_t)(G & 0xFFFFFFFFull));
         break;
@@ -480,19 +540,24 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
       if (G == 0ull) break;  // no candidate left (never for K <= N)
       if (!mine_fresh && mine > BF) {  // this slice's best might still win
         const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
-        const float g = gain_of(t);
+        const float gt = gain_of(t);
         ++my_evals;
         if (lane == 0) {
-          ub[t] = g;
+          ub[t] = gt;
           atomicOr(&fresh[t >> 5], 1u << (t & 31));
         }
+        __syncwarp();
+        rescan();
       }
       __syncthreads();
     }
-    // every thread checks the winner before anyone updates the state
-    const bool bad = pick < 0 || pick >= N || (chosen[pick >> 5] & (1u << (pick & 31))) != 0u;
+    if (threadIdx.x == 0) {  // decided once, before anyone updates the state
+      s_pick = pick;
+      s_bad = pick < 0 || pick >= N || (chosen[pick >> 5] & (1u << (pick & 31))) != 0u;
+    }
     __syncthreads();
-    if (bad) {  // never expected; block-uniform (every thread has the same pick)
+    pick = s_pick;
+    if (s_bad) {  // never expected; block-uniform
       if (threadIdx.x == 0 && atomicCAS(status, 0, CP_EDEVICE) == 0) {
         status[4] = step;
         status[5] = b;
@@ -505,19 +570,30 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
       chosen[pick >> 5] |= 1u << (pick & 31);
       order32[(size_t)b * K + step] = pick;
       if (gains) gains[(size_t)b * K + step] = ub[pick];
-      my_update_bytes += LOCAL ? 8ull * (unsigned long long)P.g : 4ull * (unsigned long long)N;
+      my_bytes += 8ull * (unsigned long long)g;
     }
-    // S <- S u {t*} (Eq. sgs_update)
-    if (!LOCAL) {
-      const float* row = Cb + (size_t)pick * ldc;
-      for (int j = threadIdx.x; j < N; j += LZ_THREADS) sm_m[j] = fminf(sm_m[j], __ldg(row + j));
-    } else {
-      const float* srow = Sb + (size_t)pick * P.g;
-      const int32_t* nb = NB + (size_t)pick * P.kk;
-      for (int k = threadIdx.x; k < P.g; k += LZ_THREADS) {
-        const int j = k == 0 ? pick : nb[k - 1];
-        sm_m[j] = fminf(sm_m[j], srow[k]);
+    // S <- S u {t*} (Eq. sgs_update) on M_g(t*), one warp a member: a target
+    // whose m drops makes every candidate on its reverse list stale
+    for (int k = w; k < g; k += LZ_WARPS) {
+      const int j = k == 0 ? pick : NB[(size_t)pick * kk + (k - 1)];
+      const float c = Sb[(size_t)pick * g + k];
+      const float mj = sm_m[j];
+      if (c < mj) {  // warp-uniform
+        __syncwarp();
+        if (lane == 0) sm_m[j] = c;
+        for (int e = roff[j] + lane; e < roff[j + 1]; e += 32) {
+          const int t = rev[e];
+          atomicAnd(&fresh[t >> 5], ~(1u << (t & 31)));
+        }
       }
+    }
+    __syncthreads();
+    // the warp that held the pick rescans; the others re-read whether their
+    // best is still exact (their bounds did not change)
+    if (w == (pick & (LZ_WARPS - 1))) {
+      rescan();
+    } else if (lane == 0) {
+      s_wfr[w] = is_fresh(s_wkey[w]);
     }
     __syncthreads();
   }
@@ -526,9 +602,8 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy(
       reinterpret_cast<unsigned char*>(status) + kCallStatsOffset);
   if (lane == 0 && my_evals) atomicAdd(&cstats[0], my_evals);
   if (threadIdx.x == 0) atomicAdd(&cstats[1], my_rounds);
-  if (lane == 0 && my_evals)
-    atomicAdd(&cstats[2], my_evals * (unsigned long long)(LOCAL ? 8 * P.g : 4 * ldc));
-  if (my_update_bytes) atomicAdd(&cstats[2], my_update_bytes);
+  if (lane == 0 && my_evals) atomicAdd(&cstats[2], my_evals * 8ull * (unsigned long long)g);
+  if (my_bytes) atomicAdd(&cstats[2], my_bytes);
   if (objective) {
     const double F = objective_sum(sm_m, sm_v, N);
     if (threadIdx.x == 0) objective[b] = F;
@@ -1085,38 +1160,41 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
   return CP_EUNSUPPORTED;
 }
 
-template <bool LOCAL>
-static int sgs_lazy_launch(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
-                           const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
-                           int32_t* order32, float* gains, double* objective, int* status,
-                           cudaStream_t s, const float* g0) {
-  const int64_t ncols = LOCAL ? N : ldc;
-  const size_t smem = sizeof(float) * (size_t)(2 * ncols + N) +
-                      2 * sizeof(uint32_t) * (size_t)((N + 31) / 32);
-  if (!LOCAL)
-    return sgs_lazy_cluster_launch(cost, ldc, v, P, B, N, K, order32, gains, objective, status, s,
-                                   g0);
-  auto fn = k_sgs_lazy<true>;
-  if (smem > 48 * 1024 &&
-      cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
-                  "launch_sgs_lazy: smem attribute") != CP_OK)
+static int sgs_local_launch(const float* slab, const int32_t* nbr, const float* v,
+                            const DevParams& P, int64_t B, int64_t N, int64_t K, int32_t* order32,
+                            float* gains, double* objective, int* status, int32_t* rev_off,
+                            int32_t* rev, cudaStream_t s) {
+  const size_t rsmem = sizeof(int) * (size_t)N;
+  if (rsmem > 48 * 1024 &&
+      cuda_status(cudaFuncSetAttribute(k_rev_build, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)rsmem),
+                  "launch_sgs_local: reverse-list smem attribute") != CP_OK)
     return CP_ECUDA;
-  fn<<<(unsigned)B, LZ_THREADS, smem, s>>>(cost, ldc, slab, nbr, v, P, (int)N, (int)K, order32,
-                                          gains, objective, status);
+  k_rev_build<<<(unsigned)B, 1024, rsmem, s>>>(nbr, (int)N, P.g, P.kk, rev_off, rev);
+  CP_TRY_STATUS(last_launch_status());
+  const size_t smem = sizeof(float) * 3 * (size_t)N + 2 * sizeof(uint32_t) * (size_t)((N + 31) / 32);
+  if (smem > 48 * 1024 &&
+      cuda_status(cudaFuncSetAttribute(k_sgs_local, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem),
+                  "launch_sgs_local: smem attribute") != CP_OK)
+    return CP_ECUDA;
+  k_sgs_local<<<(unsigned)B, LZ_THREADS, smem, s>>>(slab, nbr, v, rev_off, rev, P, (int)N, (int)K,
+                                                    order32, gains, objective, status);
   return last_launch_status();
 }
 
 int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t* nbr,
                const float* v, const DevParams& P, int64_t B, int64_t N, int64_t K,
                int32_t* order32, float* gains, double* objective, uint64_t* partials,
-               uint32_t* counters, int* status, cudaStream_t s, const float* g0) {
+               uint32_t* counters, int* status, cudaStream_t s, const float* g0,
+               int32_t* rev_off, int32_t* rev) {
   auto* part = reinterpret_cast<unsigned long long*>(partials);
   if (P.sgs_mode == 0) {
     if (P.g < N)
-      return sgs_lazy_launch<true>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
-                                   status, s, nullptr);
-    return sgs_lazy_launch<false>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,
-                                  status, s, g0);
+      return sgs_local_launch(slab, nbr, v, P, B, N, K, order32, gains, objective, status,
+                              rev_off, rev, s);
+    return sgs_lazy_cluster_launch(cost, ldc, v, P, B, N, K, order32, gains, objective, status, s,
+                                   g0);
   }
   if (P.g < N)
     return sgs_launch_impl<true>(cost, ldc, slab, nbr, v, P, B, N, K, order32, gains, objective,

@@ -298,7 +298,10 @@ def test_sgs_batch32_launch_shape(g):
                                              ("short_clip", 1500, 512, 300, 0, 3),
                                              ("long_video", 2000, 512, 400, 20, 2),
                                              ("short_clip", 777, 128, 777, 0, 1),
-                                             ("long_video", 3000, 256, 450, 0, 32)])
+                                             ("long_video", 3000, 256, 450, 0, 32),
+                                             ("long_video", 2500, 256, 600, 64, 3),
+                                             ("short_clip", 900, 128, 900, 12, 1),
+                                             ("long_video", 1200, 64, 300, 2, 2)])
 def test_sgs_lazy_equals_full_sweep(name, N, D, K, g, B):
     """Lazy evaluation only skips candidates whose earlier (upper-bound) gain
     cannot win, so it must reproduce the full sweep bit for bit."""
@@ -310,6 +313,24 @@ def test_sgs_lazy_equals_full_sweep(name, N, D, K, g, B):
     assert cp.coverprune_check(full["ws"]) == cp.CP_OK
     for k in ("kept", "order", "gains", "objective"):
         assert torch.equal(lazy[k], full[k]), k
+
+
+def test_sgs_local_duplicates_equal_full_sweep():
+    # coincident tokens share neighbourhoods and tie on gains: the reverse
+    # lists must mark every affected candidate, and ties keep the lowest index
+    rng = np.random.default_rng(7)
+    base = rng.random((150, 3)).astype(np.float32) * np.float32([6, 6, 3])
+    X = np.repeat(base, 4, axis=0)
+    f = torch.from_numpy(np.repeat(rng.standard_normal((150, 32)).astype(np.float32), 4, axis=0))
+    f = f.to(torch.bfloat16).cuda()
+    pos = torch.from_numpy(X).cuda()
+    fr = torch.from_numpy((np.arange(600) // 60).astype(np.int32)).cuda()
+    for g in (5, 33):
+        lazy = cp.coverprune_select(f, pos, fr, 200, cp.Params(g=g, sgs_mode=0))
+        full = cp.coverprune_select(f, pos, fr, 200, cp.Params(g=g, sgs_mode=1))
+        assert cp.coverprune_check(lazy["ws"]) == cp.CP_OK
+        for k in ("kept", "order", "gains", "objective"):
+            assert torch.equal(lazy[k], full[k]), (g, k)
 
 
 def test_sgs_small_edges():
