@@ -718,7 +718,7 @@ __device__ __forceinline__ float fst_cost_fold(const FstConst& k, float cosv, fl
 constexpr int FA_COLS = 1024, FA_ROWS = 32;
 
 template <bool VEC>
-__global__ void __launch_bounds__(256, 3)
+__global__ void __launch_bounds__(256, 4)
     k_fst_apply(float* __restrict__ cost, int64_t ldc, int N, const float4* __restrict__ tok,
                 const int32_t* __restrict__ frame, const SceneNorms* __restrict__ norms,
                 DevParams P, const float* __restrict__ v, float* __restrict__ g0) {
