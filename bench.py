@@ -357,30 +357,32 @@ def run_ours(args, rank, world, local_rank, raw):
         return ms / launches if ms > 0 and launches > 0 else None
 
     # the normaliser Gram (tensor cores): the pairs i <= j once, and it also
-    # stores every cosine, [B][N][ldc] fp32, for the elementwise cost pass
+    # stores their cosines (the upper triangle of [B][N][ldc] fp32) for the
+    # cost pass
     gram_ms = per_launch_ms("gram")
     gram_launches_per_step = max(prof["gram"][1] // args.steps, 1)
     gram_flops = B * N * (N + 1) * D // gram_launches_per_step
     gram_tf = gram_flops / (gram_ms / 1000.0) / 1e12 if gram_ms else None
-    # the cost pass (HBM): reads the cosines and writes the cost in place,
-    # plus each scene's token, frame and capacity columns once
+    # the cost pass (HBM): reads the cosines and writes the cost in place
     cost_ms = per_launch_ms("cost")
     cost_launches_per_step = max(prof["cost"][1] // args.steps, 1)
-    cost_bytes = (2 * B * N * ldc * 4 + B * N * (16 + 4 + 4)) // cost_launches_per_step
+    # the upper triangle of cosines read once, every cost written once, and
+    # each token's position, frame and capacity once
+    upper = B * (N * (N + 1) // 2 + N * (ldc - N)) * 4
+    cost_bytes = (upper + B * N * ldc * 4 + B * N * (16 + 4 + 4)) // cost_launches_per_step
     cost_gbs = cost_bytes / (cost_ms / 1000.0) / 1e9 if cost_ms else None
     roofline_front = {
         "normaliser_gemm": {"bound": "tensor", "kernel": "k_gram_tc", "unit": "TFLOP/s",
                             "achieved": gram_tf and round(gram_tf, 1), "peak": tf_burst,
                             "frac": gram_tf and round(gram_tf / tf_burst, 4),
                             "flops_per_launch": gram_flops,
-                            "cosine_bytes_stored_per_launch": B * N * ldc * 4
-                            // gram_launches_per_step,
+                            "cosine_bytes_stored_per_launch": upper // gram_launches_per_step,
                             "avg_launch_ms": gram_ms and round(gram_ms, 3)},
-        "fst_cost": {"bound": "hbm", "kernel": "k_fst_apply", "unit": "GB/s",
+        "fst_cost": {"bound": "hbm", "kernel": "k_fst_pair", "unit": "GB/s",
                      "achieved": cost_gbs and round(cost_gbs, 1), "peak": hbm,
                      "frac": cost_gbs and round(cost_gbs / hbm, 4),
                      "algorithmic_bytes_per_launch": cost_bytes,
-                     "traffic": read_traffic("k_fst_apply", cost_bytes),
+                     "traffic": read_traffic("k_fst_pair", cost_bytes),
                      "avg_launch_ms": cost_ms and round(cost_ms, 3)},
         "peak_source": peak_kind}
     # the line's roofline is the kernel with the largest share of the step

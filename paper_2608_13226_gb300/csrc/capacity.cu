@@ -48,8 +48,9 @@ __global__ void __launch_bounds__(256) k_capacity_r(
   if (lane == 0) r_all[(size_t)b * N + j] = P.n_cap > 0 ? acc / (float)P.n_cap : 0.0f;
 }
 
-// The same r_j from stored cosines: cos[b][j][k] (the normaliser Gram's
-// output, [B][N][ldc]) in place of the dot product, the rest identical.
+// The same r_j from stored cosines (the normaliser Gram's output, the upper
+// triangle of [B][N][ldc]: cos(j, k) at [min(j, k)][max(j, k)]) in place of
+// the dot product, the rest identical.
 // One thread per token; its n gathers fall in one row, near its own index
 // (nearest neighbours sit in the same or adjacent frames).
 __global__ void __launch_bounds__(256) k_capacity_r_cos(
@@ -69,7 +70,7 @@ __global__ void __launch_bounds__(256) k_capacity_r_cos(
   float acc = 0.0f;
   for (int q = 0; q < P.n_cap; ++q) {
     const int k = nb[q];
-    const float cosv = crow[k];
+    const float cosv = k > j ? crow[k] : cos_all[((size_t)b * N + k) * (size_t)ldc + j];
     const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
     const float dx = sqrtf(sqdist_rn(xj, yj, zj, X[3 * k], X[3 * k + 1], X[3 * k + 2]));
     const float tx = (dx - nm.x_lo) * nm.x_rinv;

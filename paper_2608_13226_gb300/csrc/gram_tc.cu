@@ -4,10 +4,11 @@
 // contraction (the cosine of Eq. fst_metrics).  k_gram_tc computes it for
 // the pairs i <= j only (the tiles on or above the diagonal) and keeps the
 // max and min cosine (the feature normaliser of Sec. 3.3); with an output
-// buffer it also stores every cosine of a pair i <= j at [i][j] and at
-// [j][i].  The FST cost of Eq. fst_cost needs the normalisers of the whole
-// scene, so it follows as one elementwise pass over the stored cosines
-// (k_fst_apply, HBM-bound), which also sums the greedy's first gains.
+// buffer it also stores every cosine of a pair i <= j at [i][j] (the upper
+// triangle).  The FST cost of Eq. fst_cost needs the normalisers of the
+// whole scene, so it follows as one pass over the stored cosines
+// (k_fst_pair, HBM-bound: each cosine read once, C(i, j) and C(j, i)
+// written), which also sums the greedy's first gains.
 //
 // Persistent clusters of two CTAs (one CTA per SM).  The two CTAs of a
 // cluster compute the row tiles 2p and 2p+1 of the same 256-column tile:
@@ -157,10 +158,6 @@ __device__ __forceinline__ void tma_load_3d_mc(const CUtensorMap* map, uint64_t*
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "h"(mask),
       "l"(policy)
       : "memory");
-}
-__device__ __forceinline__ void st_f32_policy(float* p, float v, uint64_t policy) {
-  asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" ::"l"(p), "f"(v), "l"(policy)
-               : "memory");
 }
 __device__ __forceinline__ void st_f4_policy(float* p, const float4& v, uint64_t policy) {
   asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x),
@@ -482,10 +479,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
         }
         if (a.cos_out == nullptr) continue;
-        // a chunk wholly above the diagonal (every i < j) leaves through the
-        // transpose below, one crossing it row by row for j >= i; every
-        // i < j is also stored at [j][i] (lanes hold consecutive i, so each
-        // column is one 128-byte store)
+        // only the upper triangle (j >= i) is stored: a chunk wholly above
+        // the diagonal leaves through the transpose below, one crossing it
+        // row by row; chunks below it store nothing
         const int where = j0 >= r0 + 31 ? 1 : (j0 + 31 < r0 ? -1 : 0);
         if (where == 0 && row_ok) {
 #pragma unroll
@@ -493,15 +489,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             const int j = j0 + e;
             if (j >= gi && j < a.ldc)
               a.cos_out[(sb + (size_t)gi) * (size_t)a.ldc + j] = __uint_as_float(v[e]);
-          }
-        }
-        if (where >= 0 && row_ok) {
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int j = j0 + e;
-            if (j < a.N && gi < j)
-              st_f32_policy(a.cos_out + (sb + (size_t)j) * (size_t)a.ldc + gi,
-                            __uint_as_float(v[e]), stream_out);
           }
         }
         if (where == 1) {
@@ -664,14 +651,9 @@ int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64
 }
 
 // ---------------------------------------------------------------------------
-// The FST cost from stored cosines, in place: C[i][j] = fst(cos[i][j], x, tau)
-// with the per-scene constants folded once (fst_const), and every row's
-// terms v_j max(m0 - C(i, j), 0) summed per 1024-column tile into
-// g0[b][tile][i] when g0 is given.
-// A block owns FA_COLS columns x FA_ROWS rows of one scene: each thread keeps
-// its four columns' token, frame and capacity in registers and walks the
-// rows, so the column data is read once per block (not once per element) and
-// every row of the tile is one contiguous 4 KB load and store.
+// The FST cost from the stored upper triangle of cosines, in place (one pass,
+// HBM-bound; each cosine read once, both costs of its pair written), and the
+// greedy's first-gain partial sums per 64-column tile.
 // ---------------------------------------------------------------------------
 namespace {
 
@@ -715,106 +697,217 @@ __device__ __forceinline__ float fst_cost_fold(const FstConst& k, float cosv, fl
   return fmaf(k.kL, lg, fmaf(k.kT, fmaxf(tau_s - tau_t, 0.0f), fmaf(-k.kA, cosv, k.kB)));
 }
 
-constexpr int FA_COLS = 1024, FA_ROWS = 32;
+constexpr int FP_T = 64;         // tile side
+constexpr int FP_THREADS = 256;  // 16 threads a row of a tile, 16 rows a pass
 
-template <bool VEC>
-__global__ void __launch_bounds__(256, 4)
-    k_fst_apply(float* __restrict__ cost, int64_t ldc, int N, const float4* __restrict__ tok,
-                const int32_t* __restrict__ frame, const SceneNorms* __restrict__ norms,
-                DevParams P, const float* __restrict__ v, float* __restrict__ g0) {
-  __shared__ float s_red[8][FA_ROWS];
-  const int b = blockIdx.z;
-  const int r0 = blockIdx.y * FA_ROWS;
-  const int j0 = blockIdx.x * FA_COLS + threadIdx.x * 4;
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+// The FST cost from the stored upper triangle of cosines, in place.  Block
+// (J, I, b) with I <= J takes the cosine tile of rows 64I.., columns 64J..:
+// it writes C(i, j) there and C(j, i) into the transposed tile (rows 64J..,
+// columns 64I..), both from the one cosine (the temporal term is the only
+// asymmetric part); a diagonal tile (I == J) takes its lower half from the
+// transposed upper half.  Pad columns (N <= j < ldc) get 0.  When g0 is given
+// every row's terms v_j max(m0 - C(i, j), 0) over the tile's 64 columns go to
+// g0[b][column tile][i] (each slot written by one block).  Per-scene
+// constants are folded once (fst_const).
+__global__ void __launch_bounds__(FP_THREADS, 4) k_fst_pair(
+    float* __restrict__ cost, int64_t ldc, int N, const float4* __restrict__ tok,
+    const int32_t* __restrict__ frame, const SceneNorms* __restrict__ norms, DevParams P,
+    const float* __restrict__ v, float* __restrict__ g0) {
+  const int J = blockIdx.x, I = blockIdx.y, b = blockIdx.z;
+  if (J < I) return;
+  __shared__ float sL[FP_T][FP_T + 1];  // C(j, i): rows of tile J, columns of tile I
+  __shared__ float sU[FP_T][FP_T + 1];  // diagonal tile only: the whole C tile
+  __shared__ float4 s_ti[FP_T];
+  __shared__ float s_fi[FP_T], s_vi[FP_T];
   const size_t sb = (size_t)b * N;
+  const int i0 = I * FP_T, jb = J * FP_T;
+  const bool diag = I == J;
+  const int tid = threadIdx.x;
+  const int T = gridDim.x;
+  if (tid < FP_T) {
+    const int i = i0 + tid;
+    s_ti[tid] = i < N ? __ldg(tok + sb + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    s_fi[tid] = i < N ? (float)__ldg(frame + sb + i) : 0.0f;
+    s_vi[tid] = i < N && v ? __ldg(v + sb + i) : 0.0f;
+  }
   const FstConst kf = fst_const(norms[b], P);
+  const int rl = tid >> 4, c4 = (tid & 15) * 4;  // row in the pass, first column
+  // this thread's four columns stay the same in every pass
   float4 tj[4];
-  float tauj[4], vj[4];
+  float fj[4], vj[4];
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
-    const int j = j0 + u;
-    const bool in = j < N;
-    tj[u] = in ? __ldg(tok + sb + j) : make_float4(0.f, 0.f, 0.f, 0.f);
-    tauj[u] = in ? (float)__ldg(frame + sb + j) : 0.0f;
-    vj[u] = in && v ? __ldg(v + sb + j) : 0.0f;
+    const int j = jb + c4 + u;
+    tj[u] = j < N ? __ldg(tok + sb + j) : make_float4(0.f, 0.f, 0.f, 0.f);
+    fj[u] = j < N ? (float)__ldg(frame + sb + j) : 0.0f;
+    vj[u] = j < N && v ? __ldg(v + sb + j) : 0.0f;
   }
-  const int nrow = min(FA_ROWS, N - r0);
-  for (int rr = 0; rr < nrow; rr += 4) {
-    float c[4][4];
+  __syncthreads();
+  if (!diag && (ldc & 3) == 0 && (reinterpret_cast<uintptr_t>(cost) & 15) == 0) {
+    // an off-diagonal pair with 16-byte rows (the common case): every row of
+    // tile I is a token (I < J), every column of tile I lies inside the
+    // rows, and this thread's four columns of tile J are all inside or all
+    // past the row (ldc % 4 == 0)
+    const bool cols_ld = jb + c4 < ldc;
+    const bool cols_in = jb + c4 + 3 < N;
+    const size_t step16 = (size_t)16 * (size_t)ldc;
+    float* up = cost + (sb + (size_t)(i0 + rl)) * (size_t)ldc + (jb + c4);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float* row = cost + (sb + (size_t)(r0 + rr + q)) * (size_t)ldc;
-      if (rr + q >= nrow) {
-#pragma unroll
-        for (int u = 0; u < 4; ++u) c[q][u] = 0.0f;
-      } else if (VEC) {
-        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (j0 < ldc) x = __ldcs(reinterpret_cast<const float4*>(row + j0));
-        c[q][0] = x.x, c[q][1] = x.y, c[q][2] = x.z, c[q][3] = x.w;
-      } else {
-#pragma unroll
-        for (int u = 0; u < 4; ++u) c[q][u] = j0 + u < ldc ? row[j0 + u] : 0.0f;
-      }
-    }
-    float p[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      p[q] = 0.0f;
-      if (rr + q >= nrow) continue;
-      const int i = r0 + rr + q;
-      const float4 ti = __ldg(tok + sb + i);
-      const float taui = (float)__ldg(frame + sb + i);
+    for (int pass = 0; pass < FP_T / 16; ++pass, up += step16) {
+      const int r = pass * 16 + rl;
+      float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (cols_ld) x = __ldcs(reinterpret_cast<const float4*>(up));
+      const float c[4] = {x.x, x.y, x.z, x.w};
+      const float4 ti = s_ti[r];
+      const float fi = s_fi[r];
       float o[4];
+      float part = 0.0f;
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         o[u] = 0.0f;  // pad column
-        if (j0 + u < N) {
-          o[u] = fst_cost_fold(kf, c[q][u], ti.x - tj[u].x, ti.y - tj[u].y, ti.z - tj[u].z, taui,
-                               tauj[u]);
-          p[q] = __fmaf_rn(vj[u], fmaxf(__fsub_rn(P.m0, o[u]), 0.0f), p[q]);
-        }
+        if (!cols_in && jb + c4 + u >= N) continue;
+        // fst_cost_fold for (i, j) and (j, i), sharing all but the temporal term
+        const float dx = ti.x - tj[u].x, dy = ti.y - tj[u].y, dz = ti.z - tj[u].z;
+        const float d2 = fmaxf(fmaf(dz, dz, fmaf(dy, dy, dx * dx)), 1.0e-30f);
+        const float lg = lg2_approx(fmaf(kf.kK, d2 * rsqrt_approx(d2), 1.0f));
+        const float base = fmaf(-kf.kA, c[u], kf.kB);
+        o[u] = fmaf(kf.kL, lg, fmaf(kf.kT, fmaxf(fi - fj[u], 0.0f), base));
+        sL[c4 + u][r] = fmaf(kf.kL, lg, fmaf(kf.kT, fmaxf(fj[u] - fi, 0.0f), base));
+        part = __fmaf_rn(vj[u], fmaxf(__fsub_rn(P.m0, o[u]), 0.0f), part);
       }
-      float* row = cost + (sb + (size_t)i) * (size_t)ldc;
-      if (VEC) {
-        if (j0 < ldc)
-          __stcs(reinterpret_cast<float4*>(row + j0), make_float4(o[0], o[1], o[2], o[3]));
+      if (cols_ld) __stcs(reinterpret_cast<float4*>(up), make_float4(o[0], o[1], o[2], o[3]));
+      if (g0) {  // the row's 16 threads (a half warp), in a fixed order
+#pragma unroll
+        for (int o2 = 8; o2 > 0; o2 >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o2);
+        if ((tid & 15) == 0) g0[((size_t)b * T + J) * (size_t)N + i0 + r] = part;
+      }
+    }
+    __syncthreads();
+    float* lo = cost + (sb + (size_t)(jb + rl)) * (size_t)ldc + (i0 + c4);
+#pragma unroll
+    for (int pass = 0; pass < FP_T / 16; ++pass, lo += step16) {
+      const int r = pass * 16 + rl;
+      const bool row_ok = jb + r < N;
+      float o[4];
+      float part = 0.0f;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        o[u] = sL[r][c4 + u];
+        part = __fmaf_rn(s_vi[c4 + u], fmaxf(__fsub_rn(P.m0, o[u]), 0.0f), part);
+      }
+      if (row_ok) __stcs(reinterpret_cast<float4*>(lo), make_float4(o[0], o[1], o[2], o[3]));
+      if (g0) {
+#pragma unroll
+        for (int o2 = 8; o2 > 0; o2 >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o2);
+        if ((tid & 15) == 0 && row_ok) g0[((size_t)b * T + I) * (size_t)N + jb + r] = part;
+      }
+    }
+    return;
+  }
+  // the general case (a diagonal tile, or rows that are not 16-byte aligned):
+  // rows i0 + r (r = pass * 16 + rl), columns jb + c4 .. + 3
+#pragma unroll
+  for (int pass = 0; pass < FP_T / 16; ++pass) {
+    const int r = pass * 16 + rl, i = i0 + r;
+    const bool row_ok = i < N;
+    float* row = cost + (sb + (size_t)(row_ok ? i : 0)) * (size_t)ldc;
+    const bool vec = jb + c4 + 3 < ldc && ((reinterpret_cast<uintptr_t>(row + jb + c4) & 15) == 0);
+    float c[4] = {0.f, 0.f, 0.f, 0.f};
+    if (row_ok) {
+      if (vec) {
+        const float4 x = __ldcs(reinterpret_cast<const float4*>(row + jb + c4));
+        c[0] = x.x, c[1] = x.y, c[2] = x.z, c[3] = x.w;  // below the diagonal: unused
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) c[u] = jb + c4 + u < ldc ? row[jb + c4 + u] : 0.0f;
+      }
+    }
+    const float4 ti = s_ti[r];
+    const float fi = s_fi[r];
+    float o[4];
+    float part = 0.0f;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int cl = c4 + u, j = jb + cl;
+      o[u] = 0.0f;  // pad column (or, in a diagonal tile, below the diagonal)
+      if (!row_ok || j >= N || (diag && cl < r)) continue;
+      // fst_cost_fold for (i, j) and for (j, i): the distance term and the
+      // feature term are the same (dx only changes sign), the temporal
+      // term is the one difference; the same operations, so the same bits
+      const float dx = ti.x - tj[u].x, dy = ti.y - tj[u].y, dz = ti.z - tj[u].z;
+      const float d2 = fmaxf(fmaf(dz, dz, fmaf(dy, dy, dx * dx)), 1.0e-30f);
+      const float lg = lg2_approx(fmaf(kf.kK, d2 * rsqrt_approx(d2), 1.0f));
+      const float base = fmaf(-kf.kA, c[u], kf.kB);
+      o[u] = fmaf(kf.kL, lg, fmaf(kf.kT, fmaxf(fi - fj[u], 0.0f), base));
+      if (!diag || cl > r)  // C(j, i) from the same cosine
+        sL[cl][r] = fmaf(kf.kL, lg, fmaf(kf.kT, fmaxf(fj[u] - fi, 0.0f), base));
+      part = __fmaf_rn(vj[u], fmaxf(__fsub_rn(P.m0, o[u]), 0.0f), part);
+    }
+    if (diag) {  // finished below, once the lower half is known
+#pragma unroll
+      for (int u = 0; u < 4; ++u) sU[r][c4 + u] = o[u];
+      continue;
+    }
+    if (row_ok) {
+      if (vec) {
+        __stcs(reinterpret_cast<float4*>(row + jb + c4), make_float4(o[0], o[1], o[2], o[3]));
       } else {
 #pragma unroll
         for (int u = 0; u < 4; ++u)
-          if (j0 + u < ldc) row[j0 + u] = o[u];
+          if (jb + c4 + u < ldc) row[jb + c4 + u] = o[u];
       }
     }
-    if (g0) {
-      // reduce-scatter the four rows' partials over the warp: lanes with
-      // bit 4 clear keep rows {0, 1}, set keep {2, 3}; then bit 3 picks one
-      // row; a butterfly over the low three bits completes each sum
-      const bool hb = lane & 16, mb = lane & 8;
-      const float k0 = hb ? p[2] : p[0], k1 = hb ? p[3] : p[1];
-      const float s0 = hb ? p[0] : p[2], s1 = hb ? p[1] : p[3];
-      const float q0 = k0 + __shfl_xor_sync(0xFFFFFFFFu, s0, 16);
-      const float q1 = k1 + __shfl_xor_sync(0xFFFFFFFFu, s1, 16);
-      float x = (mb ? q1 : q0) + __shfl_xor_sync(0xFFFFFFFFu, mb ? q0 : q1, 8);
-      x += __shfl_xor_sync(0xFFFFFFFFu, x, 4);
-      x += __shfl_xor_sync(0xFFFFFFFFu, x, 2);
-      x += __shfl_xor_sync(0xFFFFFFFFu, x, 1);
-      if ((lane & 7) == 0) s_red[w][rr + (hb ? 2 : 0) + (mb ? 1 : 0)] = x;
+    if (g0) {  // the row's 16 threads (a half warp), in a fixed order
+#pragma unroll
+      for (int o2 = 8; o2 > 0; o2 >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o2);
+      if ((tid & 15) == 0 && row_ok) g0[((size_t)b * T + J) * (size_t)N + i] = part;
     }
   }
-  if (g0) {
+  __syncthreads();
+  if (diag) {  // the lower half: C(i, j) for j < i is sL[i][j]
+    for (int e = tid; e < FP_T * FP_T; e += FP_THREADS) {
+      const int r = e / FP_T, cl = e % FP_T;
+      if (cl < r) sU[r][cl] = sL[r][cl];
+    }
     __syncthreads();
-    if (threadIdx.x < nrow) {
-      float sum = s_red[0][threadIdx.x];
+  }
+  // the rows of the transposed tile (I < J), or of the whole diagonal tile,
+  // from shared memory: stores and their first-gain terms (slot I)
+  float(*src)[FP_T + 1] = diag ? sU : sL;
+  const int rbase = diag ? i0 : jb;  // first row of that tile
 #pragma unroll
-      for (int ww = 1; ww < 8; ++ww) sum += s_red[ww][threadIdx.x];
-      g0[((size_t)b * gridDim.x + blockIdx.x) * (size_t)N + r0 + threadIdx.x] = sum;
+  for (int pass = 0; pass < FP_T / 16; ++pass) {
+    const int r = pass * 16 + rl, jr = rbase + r;
+    const bool row_ok = jr < N;
+    float o[4];
+    float part = 0.0f;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      o[u] = src[r][c4 + u];
+      part = __fmaf_rn(s_vi[c4 + u], fmaxf(__fsub_rn(P.m0, o[u]), 0.0f), part);
+    }
+    if (row_ok) {
+      float* row = cost + (sb + (size_t)jr) * (size_t)ldc;
+      if (i0 + c4 + 3 < ldc && ((reinterpret_cast<uintptr_t>(row + i0 + c4) & 15) == 0)) {
+        __stcs(reinterpret_cast<float4*>(row + i0 + c4), make_float4(o[0], o[1], o[2], o[3]));
+      } else {
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (i0 + c4 + u < ldc) row[i0 + c4 + u] = o[u];
+      }
+    }
+    if (g0) {  // the row's 16 threads (a half warp), in a fixed order
+#pragma unroll
+      for (int o2 = 8; o2 > 0; o2 >>= 1) part += __shfl_xor_sync(0xFFFFFFFFu, part, o2);
+      if ((tid & 15) == 0 && row_ok) g0[((size_t)b * T + I) * (size_t)N + jr] = part;
     }
   }
 }
 
-// The local neighbourhoods' costs straight from the stored cosines:
+// The local neighbourhoods' costs straight from the stored cosines (the
+// upper triangle, cos(t, j) at [min][max]):
 // slab[b][t][k] = C(t, M_g(t)[k]) with M_g(t)[0] = t and M_g(t)[k] the k-th
-// nearest other token, by the same arithmetic as k_fst_apply (the slab holds
+// nearest other token, by the same arithmetic as k_fst_pair (the slab holds
 // exactly the entries the dense cost would).  One thread per (t, k).
 __global__ void __launch_bounds__(256) k_slab_cos(const float* __restrict__ cos, int64_t ldc, int N,
                                                   int g, int kk, const int32_t* __restrict__ nbr,
@@ -830,7 +923,7 @@ __global__ void __launch_bounds__(256) k_slab_cos(const float* __restrict__ cos,
   const int j = k == 0 ? t : __ldg(nbr + (sb + t) * kk + (k - 1));
   const FstConst kf = fst_const(norms[b], P);
   const float4 ti = __ldg(tok + sb + t), tj = __ldg(tok + sb + j);
-  const float c = __ldg(cos + (sb + t) * (size_t)ldc + j);
+  const float c = __ldg(cos + (sb + min(t, j)) * (size_t)ldc + max(t, j));  // upper triangle
   slab[sb * g + i] = fst_cost_fold(kf, c, ti.x - tj.x, ti.y - tj.y, ti.z - tj.z,
                                    (float)__ldg(frame + sb + t), (float)__ldg(frame + sb + j));
 }
@@ -846,17 +939,14 @@ int launch_slab_cos(const float* cos, int64_t ldc, const int32_t* nbr, const flo
   return last_launch_status();
 }
 
-int fst_apply_slots(int64_t ldc) { return (int)((ldc + FA_COLS - 1) / FA_COLS); }
+int fst_apply_slots(int64_t ldc) { return (int)((ldc + FP_T - 1) / FP_T); }
 
 int launch_fst_apply(float* cost, int64_t ldc, int64_t B, int64_t N, const float4* tok,
                      const int32_t* frame, const SceneNorms* norms, const DevParams& P,
                      const float* v, float* g0, cudaStream_t s) {
-  const bool vec = (ldc % 4 == 0) && (reinterpret_cast<uintptr_t>(cost) % 16 == 0);
-  dim3 grid((unsigned)fst_apply_slots(ldc), (unsigned)((N + FA_ROWS - 1) / FA_ROWS), (unsigned)B);
-  if (vec)
-    k_fst_apply<true><<<grid, 256, 0, s>>>(cost, ldc, (int)N, tok, frame, norms, P, v, g0);
-  else
-    k_fst_apply<false><<<grid, 256, 0, s>>>(cost, ldc, (int)N, tok, frame, norms, P, v, g0);
+  const unsigned T = (unsigned)fst_apply_slots(ldc);
+  k_fst_pair<<<dim3(T, T, (unsigned)B), FP_THREADS, 0, s>>>(cost, ldc, (int)N, tok, frame, norms,
+                                                           P, v, g0);
   return last_launch_status();
 }
 
