@@ -792,8 +792,9 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     const float* g0 = a.g0 + (size_t)(blockIdx.x >> lgC) * a.g0_slots * a.N;
     for (int tl = threadIdx.x; tl < nown; tl += LZ_THREADS) {
       const int t = (tl << lgC) | (int)crank;
-      float sum = 0.0f;
-      for (int sl = 0; sl < a.g0_slots; ++sl) sum = __fadd_rn(sum, g0[(size_t)sl * a.N + t]);
+      float sum = 0.0f;  // the slots in order; their loads issued together
+#pragma unroll 16
+      for (int sl = 0; sl < a.g0_slots; ++sl) sum = __fadd_rn(sum, __ldg(g0 + (size_t)sl * a.N + t));
       ub[tl] = __fmaf_ru(fmaxf(sum, 0.0f), 1.00390625f, 1.0e-30f);
       if (a.use_mask)
         for (int qq = 0; qq < 4; ++qq) nzm[4 * tl + qq] = (uint16_t)0xFFFFu;
