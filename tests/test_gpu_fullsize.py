@@ -125,3 +125,40 @@ def test_lite_full_size(orc):
         t = proto_of[q]
         best = sc.min()
         assert sc[list(mem).index(t)] - best <= NEAR_TIE * max(best, 1e-12), (q, len(mem))
+
+
+@pytest.mark.parametrize("N,g", [(16384, 0), (16383, 0), (16384, 64)])
+def test_select_max_size(orc, N, g):
+    """The largest selection size (and one short of it, so the cost rows carry
+    a pad column): sampled cost entries and C(i, j) / C(j, i) pairs against
+    the oracle, and the lazy greedy equal to the full sweep bit for bit --
+    which also checks that the first-gain partial sums (one per 64 columns)
+    bound every step-0 gain from above."""
+    s = scene("long_video", 5, N=N, D=64)
+    f, pos, fr = to_dev(s)
+    p = cp.Params(g=g)
+    if g == 0:
+        out = cp.coverprune_cost(f, pos, fr)
+        torch.cuda.synchronize()
+        F = s["feats"].astype(np.float64)
+        ng = host(out["norms"])
+        nm = orc.Norms(*[float(x) for x in ng])
+        w = oracle_params(orc, p).weights
+        rng = np.random.default_rng(2)
+        S = np.concatenate([rng.integers(0, N, 4000), np.arange(0, N, 61), [N - 1, 0, N - 1]])
+        T = np.concatenate([rng.integers(0, N, 4000), np.arange(N - 1, -1, -61), [0, N - 1, N - 1]])
+        Cg = host(out["cost"])
+        Co = orc.cost_pairs(F, s["pos"], s["frame"], w, nm, S, T)
+        assert_cost_close(Cg[S, T], Co, "bf16")
+        Co_t = orc.cost_pairs(F, s["pos"], s["frame"], w, nm, T, S)
+        assert_cost_close(Cg[T, S], Co_t, "bf16", "transposed cost")
+        del out, Cg
+    K = 300
+    lazy = cp.coverprune_select(f, pos, fr, K, cp.Params(g=g, sgs_mode=0))
+    full = cp.coverprune_select(f, pos, fr, K, cp.Params(g=g, sgs_mode=1))
+    assert cp.coverprune_check(lazy["ws"]) == cp.CP_OK
+    assert cp.coverprune_check(full["ws"]) == cp.CP_OK
+    for k in ("kept", "order", "gains", "objective"):
+        assert torch.equal(lazy[k], full[k]), k
+    kept = host(lazy["kept"])
+    assert np.all(np.diff(kept) > 0) and kept[0] >= 0 and kept[-1] < N
