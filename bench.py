@@ -19,6 +19,7 @@ cores on a bounded sample of the same workload, scaled to scenes per second.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import datetime
 import json
 import math
@@ -470,39 +471,47 @@ def run_ours(args, rank, world, local_rank, raw):
              "stages_ms": {k: round(v[0] / args.steps, 3) for k, v in gprof.items() if v[0] > 0}}
     del wsg
 
-    # CoverPrune-Lite on the same batch
-    wsl = cp.workspace(cp.CP_OP_LITE, B, N, D, K, cp.CP_BF16, prm, dev)
-    lite_out = {"kept": torch.empty(B, K, dtype=torch.int64, device=dev)}
-    for _ in range(args.warmup):
-        cp.coverprune_lite_select(feats, pos, fr, K, prm, group_start=False, objective=False,
-                                  ws=wsl, out=lite_out)
-    barrier()
-    cp.coverprune_profile_read()
-    cp.coverprune_profile_enable(True)
-    a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    for _ in range(args.steps):
-        cp.coverprune_lite_select(feats, pos, fr, K, prm, group_start=False, objective=False,
-                                  ws=wsl, out=lite_out)
-    b_.record(stream)
-    barrier()
-    cp.coverprune_profile_enable(False)
-    lprof = cp.coverprune_profile_read()
-    lite_ms = max_over_ranks(a.elapsed_time(b_) / args.steps)
-    lat_l = []
-    for i in range(6):
+    # CoverPrune-Lite on the same batch: with the min-max feature normaliser
+    # (the Gram over all pairs runs first), and with the bounded one (d_f / 2,
+    # no all-pairs pass)
+    def measure_lite(prm_l):
+        wsl = cp.workspace(cp.CP_OP_LITE, B, N, D, K, cp.CP_BF16, prm_l, dev)
+        lite_out = {"kept": torch.empty(B, K, dtype=torch.int64, device=dev)}
+        for _ in range(args.warmup):
+            cp.coverprune_lite_select(feats, pos, fr, K, prm_l, group_start=False,
+                                      objective=False, ws=wsl, out=lite_out)
+        barrier()
+        cp.coverprune_profile_read()
+        cp.coverprune_profile_enable(True)
         a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        cp.coverprune_lite_select(feats[0], pos[0], fr[0], K, prm, group_start=False,
-                                  objective=False)
+        for _ in range(args.steps):
+            cp.coverprune_lite_select(feats, pos, fr, K, prm_l, group_start=False,
+                                      objective=False, ws=wsl, out=lite_out)
         b_.record(stream)
-        torch.cuda.synchronize()
-        if i >= 2:
-            lat_l.append(a.elapsed_time(b_))
-    lite = {"scenes_per_s": B * world / (lite_ms / 1000.0), "ms_per_step": round(lite_ms, 3),
-            "latency_ms": round(statistics.median(lat_l), 3),
-            "stages_ms": {k: round(v[0] / args.steps, 3) for k, v in lprof.items() if v[0] > 0}}
-    del wsl
+        barrier()
+        cp.coverprune_profile_enable(False)
+        lprof = cp.coverprune_profile_read()
+        lite_ms = max_over_ranks(a.elapsed_time(b_) / args.steps)
+        lat_l = []
+        for i in range(6):
+            a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            cp.coverprune_lite_select(feats[0], pos[0], fr[0], K, prm_l, group_start=False,
+                                      objective=False)
+            b_.record(stream)
+            torch.cuda.synchronize()
+            if i >= 2:
+                lat_l.append(a.elapsed_time(b_))
+        del wsl
+        return {"scenes_per_s": B * world / (lite_ms / 1000.0), "ms_per_step": round(lite_ms, 3),
+                "latency_ms": round(statistics.median(lat_l), 3),
+                "stages_ms": {k: round(v[0] / args.steps, 3) for k, v in lprof.items()
+                              if v[0] > 0}}
+
+    lite = measure_lite(prm)
+    lite_bounded = measure_lite(dataclasses.replace(prm, norm_mode=1))
+    lite_bounded["norm_mode"] = "bounded feature normaliser (d_f / 2): no all-pairs Gram"
 
     # end to end through the C ABI with host buffers, as a serving loop runs
     # it: every step uploads its inputs from pinned host memory (on a copy
@@ -591,7 +600,7 @@ def run_ours(args, rank, world, local_rank, raw):
                        "generator": "paper_2608_13226_gb300.scenes long_video, seeds "
                                     f"{rank * B}..{rank * B + B - 1} per rank"},
             "latency_ms": round(latency_ms, 3),
-            "lite": lite, "local_sgs": local, "roofline": roofline, "roofline_sgs": roofline_sgs,
+            "lite": lite, "lite_bounded": lite_bounded, "local_sgs": local, "roofline": roofline, "roofline_sgs": roofline_sgs,
             "roofline_front": roofline_front, "sgs_full_sweep": sweep,
             "stages_ms": stages, "gpu_launches": gpu_launches, "e2e": e2e,
             "clocks": clocks, "cpu_baseline": cpu}

@@ -109,6 +109,16 @@ typedef enum {
  *                                   current one, so only candidates whose
  *                                   bound could still win are re-evaluated;
  *                                   default), 1 = every gain every step
+ *   norm_mode                       feature normaliser of Eq. fst_cost: 0 =
+ *                                   min-max of d_f over all ordered pairs of
+ *                                   the scene (Sec. 3.3; default); 1 =
+ *                                   bounded, d_f / 2 (d_f = 1 - cos lies in
+ *                                   [0, 2]), which needs no all-pairs pass, so
+ *                                   Lite runs without the N^2 D Gram (the
+ *                                   complexity Sec. 4 states).  The spatial
+ *                                   and temporal normalisers are the same in
+ *                                   both.  The two agree whenever the scene
+ *                                   holds a pair with cos = -1.
  */
 typedef struct {
   uint32_t struct_size; /* = sizeof(cp_params); set by cp_default_params */
@@ -122,6 +132,7 @@ typedef struct {
   float m0;
   float timeout_ms;
   int32_t sgs_mode;
+  int32_t norm_mode;
 } cp_params;
 
 /* Fills *p with the defaults listed above.  Host only; p must not be NULL. */

@@ -110,6 +110,8 @@ def _load():
         lib.orc_set_threads.argtypes = [C.c_int]
         lib.orc_get_threads.restype = C.c_int
         lib.orc_normalisers.argtypes = [_I64, _I64, _P, _P, _P, C.POINTER(_Norms)]
+        lib.orc_normalisers_mode.argtypes = [_I64, _I64, _P, _P, _P, C.c_int,
+                                             C.POINTER(_Norms)]
         lib.orc_cost_rows.argtypes = [_I64, _I64, _P, _P, _P, C.POINTER(_Weights),
                                       C.POINTER(_Norms), _I64, _I64, _P]
         lib.orc_cost_pairs.argtypes = [_I64, _I64, _P, _P, _P, C.POINTER(_Weights),
@@ -124,7 +126,7 @@ def _load():
         lib.orc_lite_groups.argtypes = [_I64, _I64, _P, _P, _P, _P]
         lib.orc_lite_select.argtypes = [_I64, _I64, _P, _P, _P, C.POINTER(_Weights),
                                         C.POINTER(_Norms), _P, _P, _P, _I64, _P, _P, _P]
-        for fn in ("orc_normalisers", "orc_cost_rows", "orc_cost_pairs", "orc_knn_others",
+        for fn in ("orc_normalisers", "orc_normalisers_mode", "orc_cost_rows", "orc_cost_pairs", "orc_knn_others",
                    "orc_capacity", "orc_objective", "orc_sgs", "orc_morton",
                    "orc_lite_groups", "orc_lite_select"):
             getattr(lib, fn).restype = C.c_int
@@ -167,13 +169,15 @@ def get_threads() -> int:
 # Cost and capacity
 # --------------------------------------------------------------------------
 
-def normalisers(F, X, tau) -> Norms:
-    """Min and max of d_f, d_x, d_tau over all ordered pairs (Sec. 3.3)."""
+def normalisers(F, X, tau, norm_mode: int = 0) -> Norms:
+    """Min and max of d_f, d_x, d_tau over all ordered pairs (Sec. 3.3);
+    norm_mode 1 takes the bounds [0, 2] of d_f = 1 - cos instead of its
+    measured range (the bounded feature normaliser)."""
     F, X, tau = _f64(F), _pos(X), _tau(tau)
     N, D = F.shape
     out = _Norms()
-    _check(_load().orc_normalisers(N, D, _ptr(F), _ptr(X), _ptr(tau), C.byref(out)),
-           "normalisers")
+    _check(_load().orc_normalisers_mode(N, D, _ptr(F), _ptr(X), _ptr(tau), int(norm_mode),
+                                        C.byref(out)), "normalisers")
     return Norms(out.f_lo, out.f_hi, out.x_lo, out.x_hi, out.tau_lo, out.tau_hi)
 
 
@@ -333,13 +337,15 @@ class Params:
     """Method parameters.  n_cap = |N_n| (capacity neighbours), g = |M_g|
     (0 = all tokens), capacity_mode 0 = FST capacity, 1 = uniform,
     m0 = initial coverage cost (<= 0 means lambda_f + lambda_x + lambda_tau),
-    voxel = Morton cell in metres."""
+    voxel = Morton cell in metres, norm_mode 0 = min-max feature normaliser,
+    1 = bounded (d_f / 2)."""
     weights: Weights = None
     n_cap: int = 8
     g: int = 0
     capacity_mode: int = 0
     m0: float = 0.0
     voxel: float = 0.2
+    norm_mode: int = 0
 
     def __post_init__(self):
         if self.weights is None:
@@ -353,7 +359,7 @@ class Params:
 def prepare(F, X, tau, prm: Params) -> dict:
     """Normalisers, capacity neighbours and capacity of one scene."""
     N = np.asarray(F).shape[0]
-    nm = normalisers(F, X, tau)
+    nm = normalisers(F, X, tau, prm.norm_mode)
     n = min(prm.n_cap, N - 1)
     g = prm.g if 0 < prm.g < N else N
     k = max(n, g - 1) if g < N else n

@@ -174,9 +174,15 @@ static double fst_cost(const double* F, const double* nrm, int64_t D,
 /* Normalisers: min and max of each discrepancy over all ordered pairs */
 /* ------------------------------------------------------------------ */
 
-int orc_normalisers(int64_t N, int64_t D, const double* F, const float* X,
-                    const int32_t* tau, orc_norms* out) {
+/* feat_mode 0: the range of d_f over all ordered pairs, as for d_x and
+ * d_tau (Sec. 3.3).  feat_mode 1, the bounded feature normaliser: d_f =
+ * 1 - cos always lies in [0, 2] (cos is clamped to [-1, 1]), so that range
+ * stands in for the measured one and d_f is not visited; d_x and d_tau keep
+ * their measured ranges. */
+int orc_normalisers_mode(int64_t N, int64_t D, const double* F, const float* X,
+                         const int32_t* tau, int feat_mode, orc_norms* out) {
   if (N < 1 || D < 1 || !F || !X || !tau || !out) return ORC_EINVAL;
+  if (feat_mode != 0 && feat_mode != 1) return ORC_EINVAL;
   double* nrm = all_norms(F, N, D);
   if (!nrm) return ORC_ENOMEM;
   double f_lo = INFINITY, f_hi = -INFINITY;
@@ -189,10 +195,12 @@ int orc_normalisers(int64_t N, int64_t D, const double* F, const float* X,
   for (int64_t s = 0; s < N; ++s) {
     for (int64_t t = 0; t < N; ++t) {
       if (t >= s) {
-        double df = disc_f(F, nrm, D, s, t);
+        if (feat_mode == 0) {
+          double df = disc_f(F, nrm, D, s, t);
+          if (df < f_lo) f_lo = df;
+          if (df > f_hi) f_hi = df;
+        }
         double dx = disc_x(X, s, t);
-        if (df < f_lo) f_lo = df;
-        if (df > f_hi) f_hi = df;
         if (dx < x_lo) x_lo = dx;
         if (dx > x_hi) x_hi = dx;
       }
@@ -202,10 +210,19 @@ int orc_normalisers(int64_t N, int64_t D, const double* F, const float* X,
     }
   }
   free(nrm);
+  if (feat_mode == 1) {
+    f_lo = 0.0;
+    f_hi = 2.0;
+  }
   out->f_lo = f_lo; out->f_hi = f_hi;
   out->x_lo = x_lo; out->x_hi = x_hi;
   out->tau_lo = t_lo; out->tau_hi = t_hi;
   return ORC_OK;
+}
+
+int orc_normalisers(int64_t N, int64_t D, const double* F, const float* X,
+                    const int32_t* tau, orc_norms* out) {
+  return orc_normalisers_mode(N, D, F, X, tau, 0, out);
 }
 
 /* ------------------------------------------------------------------ */

@@ -47,7 +47,7 @@ class _CpParams(C.Structure):
                 ("alpha_f", C.c_float), ("alpha_x", C.c_float), ("alpha_tau", C.c_float),
                 ("n_cap", C.c_int32), ("g", C.c_int32), ("capacity_mode", C.c_int32),
                 ("voxel_m", C.c_float), ("m0", C.c_float), ("timeout_ms", C.c_float),
-                ("sgs_mode", C.c_int32)]
+                ("sgs_mode", C.c_int32), ("norm_mode", C.c_int32)]
 
 
 class _CallStats(C.Structure):
@@ -73,6 +73,7 @@ class Params:
     m0: float = 0.0
     timeout_ms: float = 2000.0
     sgs_mode: int = 0
+    norm_mode: int = 0
 
     def _c(self) -> _CpParams:
         p = _CpParams()

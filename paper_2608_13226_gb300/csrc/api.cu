@@ -154,6 +154,7 @@ static int check_params(const cp_params* p) {
   if (p->n_cap < 0 || p->g < 0) return CP_EINVAL;
   if (p->capacity_mode != 0 && p->capacity_mode != 1) return CP_EINVAL;
   if (p->sgs_mode != 0 && p->sgs_mode != 1) return CP_EINVAL;
+  if (p->norm_mode != 0 && p->norm_mode != 1) return CP_EINVAL;
   return CP_OK;
 }
 
@@ -184,6 +185,7 @@ static DevParams dev_params(const cp_params* p, int64_t N) {
   d.kk = d.g < N ? (d.n_cap > d.g - 1 ? d.n_cap : d.g - 1) : d.n_cap;
   d.cap_mode = p->capacity_mode;
   d.sgs_mode = p->sgs_mode;
+  d.norm_mode = p->norm_mode;
   d.timeout_ns = (uint64_t)((double)p->timeout_ms * 1.0e6);
   return d;
 }
@@ -304,14 +306,18 @@ static int run_front(const void* feats, int dtype, const float* pos, const int32
       CP_TRY(launch_knn(pos, at<float4>(ws, pl.tok), B, N, d.kk, at<int32_t>(ws, pl.nbr), stats,
                         s));
   }
-  {
+  // the Gram gives the min-max feature normaliser and, for bf16 inputs, the
+  // stored cosines; with the bounded normaliser and no cosines to store
+  // (Lite, or fp32 inputs) it does not run
+  cos_out = dtype == CP_BF16 ? cos_out : nullptr;
+  if (d.norm_mode == 0 || cos_out) {
     Stage st(CP_STAGE_GRAM, s);
     CP_TRY(launch_gram_minmax(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), B, N,
-                              D, stats, status, d.timeout_ns, s,
-                              dtype == CP_BF16 ? cos_out : nullptr, ldc));
+                              D, stats, status, d.timeout_ns, s, cos_out, ldc));
   }
   Stage st(CP_STAGE_PREP, s);
-  CP_TRY(launch_finalize_norms(stats, B, at<SceneNorms>(ws, pl.norms), norms_out, s));
+  CP_TRY(launch_finalize_norms(stats, B, d.norm_mode, at<SceneNorms>(ws, pl.norms), norms_out,
+                               s));
   return CP_OK;
 }
 
@@ -348,6 +354,7 @@ void cp_default_params(cp_params* p) {
   p->m0 = 0.0f;
   p->timeout_ms = 2000.0f;
   p->sgs_mode = 0;
+  p->norm_mode = 0;
 }
 
 int64_t coverprune_budget(double R, int64_t N) {

@@ -21,6 +21,7 @@ struct DevParams {
   int kk;      // neighbours stored per token = max(n_cap, g-1) (g < N) or n_cap
   int cap_mode;
   int sgs_mode;  // 0 = lazy evaluation of gains, 1 = every gain every step
+  int norm_mode;  // feature normaliser: 0 = min-max over all pairs, 1 = d_f / 2
   uint64_t timeout_ns;
 };
 
@@ -115,8 +116,9 @@ int launch_gram_minmax(const void* feats, int dtype, const float* inv, const flo
                        float* cos_out = nullptr, int64_t ldc = 0);
 // Scene diameter sqrt(max d^2) from stats into out[b].
 int launch_diameter(const SceneStats* stats, int64_t B, float* out, cudaStream_t s);
-// Normalisers from stats.  Optionally also the public [B, 6] float copy.
-int launch_finalize_norms(const SceneStats* stats, int64_t B, SceneNorms* norms,
+// Normalisers from stats (norm_mode 1: the feature range is [0, 2] instead of
+// the Gram's extremes).  Optionally also the public [B, 6] float copy.
+int launch_finalize_norms(const SceneStats* stats, int64_t B, int norm_mode, SceneNorms* norms,
                           float* norms_out, cudaStream_t s);
 // K3 for fp32 features: the FST cost C[b][s][t] into cost + b*N*ldc + s*ldc
 // + t for t < N; columns N <= t < ldc are written as 0.  (bf16 features:

@@ -919,15 +919,17 @@ int launch_diameter(const SceneStats* stats, int64_t B, float* out, cudaStream_t
 // ---------------------------------------------------------------------------
 // Normalisers from the reduced statistics.
 // ---------------------------------------------------------------------------
-__global__ void k_finalize_norms(const SceneStats* stats, int B, SceneNorms* norms,
-                                 float* norms_out) {
+__global__ void k_finalize_norms(const SceneStats* stats, int B, int norm_mode,
+                                 SceneNorms* norms, float* norms_out) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   const SceneStats st = stats[b];
   SceneNorms nm;
   const float cmax = key2f(st.cos_max_key), cmin = key2f(st.cos_min_key);
-  nm.f_lo = 1.0f - cmax;
-  nm.f_hi = 1.0f - cmin;
+  // min-max over all pairs (the Gram's extremes), or the bounds of
+  // d_f = 1 - cos itself, [0, 2]
+  nm.f_lo = norm_mode == 1 ? 0.0f : 1.0f - cmax;
+  nm.f_hi = norm_mode == 1 ? 2.0f : 1.0f - cmin;
   nm.x_lo = 0.0f;  // diagonal pairs: d_x(j, j) = 0
   nm.x_hi = sqrtf(__uint_as_float(st.d2_max_bits));
   nm.t_lo = 0.0f;  // d_tau(j, j) = 0 and d_tau >= 0
@@ -944,9 +946,10 @@ __global__ void k_finalize_norms(const SceneStats* stats, int B, SceneNorms* nor
   }
 }
 
-int launch_finalize_norms(const SceneStats* stats, int64_t B, SceneNorms* norms,
+int launch_finalize_norms(const SceneStats* stats, int64_t B, int norm_mode, SceneNorms* norms,
                           float* norms_out, cudaStream_t s) {
-  k_finalize_norms<<<(unsigned)((B + 127) / 128), 128, 0, s>>>(stats, (int)B, norms, norms_out);
+  k_finalize_norms<<<(unsigned)((B + 127) / 128), 128, 0, s>>>(stats, (int)B, norm_mode, norms,
+                                                               norms_out);
   return last_launch_status();
 }
 

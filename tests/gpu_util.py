@@ -37,7 +37,7 @@ def oracle_params(orc, p: cp.Params):
     w = orc.Weights(p.lambda_f, p.lambda_x, p.lambda_tau, p.kappa, p.alpha_f, p.alpha_x,
                     p.alpha_tau)
     return orc.Params(weights=w, n_cap=p.n_cap, g=p.g, capacity_mode=p.capacity_mode,
-                      m0=p.m0, voxel=p.voxel_m)
+                      m0=p.m0, voxel=p.voxel_m, norm_mode=p.norm_mode)
 
 
 def assert_cost_close(Cg, Co, dtype, what="cost"):

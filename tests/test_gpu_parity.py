@@ -114,7 +114,7 @@ def _cost_case(orc, s, prm=cp.Params()):
     out = cp.coverprune_cost(f, pos, fr, prm)
     torch.cuda.synchronize()
     F = f64(s)
-    nm = orc.normalisers(F, s["pos"], s["frame"])
+    nm = orc.normalisers(F, s["pos"], s["frame"], prm.norm_mode)
     op = oracle_params(orc, prm)
     Co = orc.cost_matrix(F, s["pos"], s["frame"], op.weights, nm)
     _, vo = orc.capacity(F, s["pos"], s["frame"], op.weights, nm, prm.n_cap, mode=prm.capacity_mode)
@@ -169,6 +169,38 @@ def test_cost_ablation_weights(orc):
     assert_capacity_close(host(out["capacity"]), vo, "bf16")
     out1, _, _, vo1 = _cost_case(orc, s, cp.Params(capacity_mode=1))
     np.testing.assert_allclose(host(out1["capacity"]), 1.0 / 500, rtol=1e-7)
+
+
+@pytest.mark.parametrize("name,N,D,dtype", [("tiny", 1024, 256, "f32"),
+                                            ("long_video", 777, 512, "bf16")])
+def test_cost_bounded_normaliser(orc, name, N, D, dtype):
+    """norm_mode 1: the feature term is d_f / 2; the fp32 path runs without
+    the Gram, the bf16 path still takes its cosines from it."""
+    s = scene(name, 5, N=N, D=D)
+    prm = cp.Params(norm_mode=1)
+    out, nm, Co, vo = _cost_case(orc, s, prm)
+    ng = host(out["norms"])
+    assert ng[0] == 0.0 and ng[1] == 2.0
+    np.testing.assert_allclose(ng, [nm.f_lo, nm.f_hi, nm.x_lo, nm.x_hi, nm.tau_lo, nm.tau_hi],
+                               rtol=1e-5, atol=1e-6)
+    assert_cost_close(host(out["cost"]), Co, dtype)
+    assert_capacity_close(host(out["capacity"]), vo, dtype)
+    # the min-max cost of the same scene differs (its feature range is < 2)
+    ref = cp.coverprune_cost(*to_dev(s), cp.Params(), capacity=False, norms=False)["cost"]
+    assert not torch.equal(ref, out["cost"])
+
+
+def test_sgs_bounded_normaliser_teacher_forced(orc):
+    s = scene("short_clip", 6, N=999, D=512)
+    K = 200
+    prm = cp.Params(norm_mode=1)
+    sel, cst = _select_case(orc, s, K, prm)
+    order = host(sel["order"])
+    check_sgs_teacher_forced(orc, host(cst["cost"]).astype(np.float64),
+                             host(cst["capacity"]).astype(np.float64), order, host(sel["gains"]),
+                             float(host(sel["objective"])), 3.0, 0, None)
+    ora = orc.select(f64(s), s["pos"], s["frame"], K, oracle_params(orc, prm))
+    check_sgs_end_to_end(orc, ora, order, host(sel["kept"]), 3.0, 0)
 
 
 def test_cost_degenerate_scenes(orc):
@@ -358,7 +390,7 @@ def _lite_check(orc, s, K, prm, dtype):
     b, _ = orc.lite_groups(vg, perm, K)
     np.testing.assert_array_equal(host(lt["group_start"]), b)  # exact integer grouping
     F = f64(s)
-    nm = orc.normalisers(F, s["pos"], s["frame"])
+    nm = orc.normalisers(F, s["pos"], s["frame"], prm.norm_mode)
     op = oracle_params(orc, prm)
     proto, score, obj = orc.lite_select(F, s["pos"], s["frame"], op.weights, nm,
                                         vg.astype(np.float64), perm, b)
@@ -389,6 +421,14 @@ def test_lite_parity(orc, name, N, D, K):
     dtype = s["dtype"]
     near = _lite_check(orc, s, K, cp.Params(), dtype)
     print(f"lite {name}: near-tie prototype differences {near}/{K}")
+
+
+@pytest.mark.parametrize("name,N,D,K", [("tiny", 1024, 256, 102), ("long_video", 1500, 512, 150)])
+def test_lite_bounded_normaliser(orc, name, N, D, K):
+    """Lite with the bounded feature normaliser (no Gram pass at all)."""
+    s = scene(name, 2, N=N, D=D)
+    near = _lite_check(orc, s, K, cp.Params(norm_mode=1), s["dtype"])
+    print(f"lite bounded {name}: near-tie prototype differences {near}/{K}")
 
 
 def test_lite_edges(orc):

@@ -58,6 +58,59 @@ def test_worked_example_norms_and_cost(orc):
     np.testing.assert_allclose(Cm, want, atol=1e-12, rtol=0)
 
 
+def test_worked_example_bounded_normaliser(orc):
+    """The bounded feature normaliser (d_f / 2) on the worked example: hand
+    values of the norms, the cost matrix and the uniform SGS."""
+    F, X, tau = ex_inputs()
+    bn = GOLD["bounded_norm"]
+    nm = orc.normalisers(F, X, tau, norm_mode=1)
+    for k, e in bn["norms"].items():
+        assert getattr(nm, k) == pytest.approx(ev(e), abs=1e-12), k
+    Cm = orc.cost_matrix(F, X, tau, orc.Weights(kappa=GOLD["kappa"]), nm)
+    want = np.array([[ev(e) for e in row] for row in bn["cost"]])
+    np.testing.assert_allclose(Cm, want, atol=1e-12, rtol=0)
+    v = np.full(3, 1.0 / 3.0)
+    M0 = GOLD["M0"]
+    for t, e in enumerate(bn["uniform_step1_gains"]):
+        assert M0 - orc.objective(Cm, v, [t], M0) == pytest.approx(ev(e), abs=1e-12)
+    res = orc.sgs(Cm, v, 2, M0)
+    assert list(res["order"]) == bn["uniform_K2_order"]
+    after = bn["uniform_step2_gains_after_1"]
+    assert res["best_gain"][1] == pytest.approx(ev(after["2"]), abs=1e-12)
+    assert res["second"][1] == pytest.approx(ev(after["0"]), abs=1e-12)
+    assert res["F"] == pytest.approx(ev(bn["uniform_K2_F"]), abs=1e-12)
+    # end to end through the driver's parameter
+    prm = orc.Params(weights=orc.Weights(kappa=GOLD["kappa"]), capacity_mode=1, m0=M0,
+                     norm_mode=1)
+    r = orc.select(F, X, tau, 2, prm)
+    assert list(r["order"]) == bn["uniform_K2_order"]
+
+
+def test_bounded_normaliser_equals_minmax_with_antipodal_pair(orc):
+    """A scene holding f and -f has min cos = -1, so the measured feature
+    range is [0, 2] and both normalisers give the same cost; the spatial and
+    temporal ranges never depend on the mode."""
+    rng = np.random.default_rng(11)
+    F, X, tau = rand_scene(rng, 40)
+    F[7] = -F[3]
+    a = orc.normalisers(F, X, tau, norm_mode=0)
+    b = orc.normalisers(F, X, tau, norm_mode=1)
+    assert a.f_lo == pytest.approx(0.0, abs=1e-12) and a.f_hi == pytest.approx(2.0, abs=1e-12)
+    assert (a.x_lo, a.x_hi, a.tau_lo, a.tau_hi) == (b.x_lo, b.x_hi, b.tau_lo, b.tau_hi)
+    w = orc.Weights()
+    np.testing.assert_allclose(orc.cost_matrix(F, X, tau, w, a), orc.cost_matrix(F, X, tau, w, b),
+                               atol=1e-12, rtol=0)
+    # without the antipodal pair the feature term is scaled by range / 2
+    F2, X2, tau2 = rand_scene(np.random.default_rng(12), 40)
+    a2 = orc.normalisers(F2, X2, tau2, norm_mode=0)
+    b2 = orc.normalisers(F2, X2, tau2, norm_mode=1)
+    assert a2.f_hi < 2.0 and (b2.f_lo, b2.f_hi) == (0.0, 2.0)
+    wf = orc.Weights(lambda_x=0.0, lambda_tau=0.0)
+    Ca = orc.cost_matrix(F2, X2, tau2, wf, a2)
+    Cb = orc.cost_matrix(F2, X2, tau2, wf, b2)
+    np.testing.assert_allclose(Cb, Ca * (a2.f_hi - a2.f_lo) / 2.0, atol=1e-12, rtol=0)
+
+
 def test_worked_example_uniform_sgs(orc):
     F, X, tau = ex_inputs()
     w = orc.Weights(kappa=GOLD["kappa"])
