@@ -5,16 +5,23 @@
 namespace cp {
 
 // r_j = (1/n) sum_{k in N_n(j)} alpha_f d^_f(j,k) + alpha_x d^_x(j,k) + alpha_tau d^_tau(j,k)
-// One warp per token; the dot products run over 16-byte feature vectors.
+// One block per token, one warp per neighbour (warp w takes k = N_n(j)[q]
+// for q = w, w + warps, ...): the warps read the token's own row together,
+// so L1 serves it once for all of them, and each reads one neighbour row.
+// The dot products run over 16-byte feature vectors; the terms are summed in
+// neighbour order by one thread.
+constexpr int CAP_WARPS = 8;
 template <typename T>
-__global__ void __launch_bounds__(256) k_capacity_r(
+__global__ void __launch_bounds__(32 * CAP_WARPS) k_capacity_r(
     const T* __restrict__ F_all, const float* __restrict__ inv_all, const float* __restrict__ pos_all,
     const int32_t* __restrict__ frame_all, const SceneNorms* __restrict__ norms,
     const int32_t* __restrict__ nbr_all, DevParams P, int N, int D, float* __restrict__ r_all) {
-  const int j = blockIdx.x * 8 + (threadIdx.x >> 5);
+  constexpr int CHUNK = 256;
+  __shared__ float s_term[CHUNK];  // the terms of neighbours q0 .. q0 + CHUNK - 1
+  const int j = blockIdx.x;
   const int b = blockIdx.y;
-  const int lane = threadIdx.x & 31;
-  if (j >= N) return;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nw = (int)(blockDim.x >> 5);
   const T* F = F_all + (size_t)b * N * D;
   const float* inv = inv_all + (size_t)b * N;
   const float* X = pos_all + (size_t)b * N * 3;
@@ -23,29 +30,36 @@ __global__ void __launch_bounds__(256) k_capacity_r(
   const SceneNorms nm = norms[b];
   constexpr int V = Vec16<T>::n;
   const T* fj = F + (size_t)j * D;
-  float acc = 0.0f;
-  for (int q = 0; q < P.n_cap; ++q) {
-    const int k = nb[q];
-    const T* fk = F + (size_t)k * D;
-    float dot = 0.0f;
-    for (int d = lane * V; d < D; d += 32 * V) {
-      float a[V], c[V];
-      Vec16<T>::load(fj + d, a);
-      Vec16<T>::load(fk + d, c);
+  float acc = 0.0f;  // thread 0's running sum, in neighbour order
+  for (int q0 = 0; q0 < P.n_cap; q0 += CHUNK) {
+    const int qn = min(CHUNK, P.n_cap - q0);
+    for (int qq = w; qq < qn; qq += nw) {
+      const int k = __ldg(nb + q0 + qq);
+      const T* fk = F + (size_t)k * D;
+      float dot = 0.0f;
+      for (int d = lane * V; d < D; d += 32 * V) {
+        float a[V], c[V];
+        Vec16<T>::load(fj + d, a);
+        Vec16<T>::load(fk + d, c);
 #pragma unroll
-      for (int i = 0; i < V; ++i) dot = fmaf(a[i], c[i], dot);
+        for (int i = 0; i < V; ++i) dot = fmaf(a[i], c[i], dot);
+      }
+      dot = warp_sum(dot);
+      const float cosv = clamp_cos(dot * inv[j] * inv[k]);
+      const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
+      const float dx = sqrtf(sqdist_rn(X[3 * j], X[3 * j + 1], X[3 * j + 2], X[3 * k],
+                                       X[3 * k + 1], X[3 * k + 2]));
+      const float tx = (dx - nm.x_lo) * nm.x_rinv;
+      const int dt = TAU[j] - TAU[k];
+      const float tt = dt > 0 ? (float)dt * nm.t_rinv : 0.0f;
+      if (lane == 0) s_term[qq] = P.alpha_f * tf + P.alpha_x * tx + P.alpha_tau * tt;
     }
-    dot = warp_sum(dot);
-    const float cosv = clamp_cos(dot * inv[j] * inv[k]);
-    const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
-    const float dx = sqrtf(sqdist_rn(X[3 * j], X[3 * j + 1], X[3 * j + 2], X[3 * k], X[3 * k + 1],
-                                     X[3 * k + 2]));
-    const float tx = (dx - nm.x_lo) * nm.x_rinv;
-    const int dt = TAU[j] - TAU[k];
-    const float tt = dt > 0 ? (float)dt * nm.t_rinv : 0.0f;
-    acc += P.alpha_f * tf + P.alpha_x * tx + P.alpha_tau * tt;
+    __syncthreads();
+    if (threadIdx.x == 0)
+      for (int qq = 0; qq < qn; ++qq) acc += s_term[qq];
+    __syncthreads();
   }
-  if (lane == 0) r_all[(size_t)b * N + j] = P.n_cap > 0 ? acc / (float)P.n_cap : 0.0f;
+  if (threadIdx.x == 0) r_all[(size_t)b * N + j] = P.n_cap > 0 ? acc / (float)P.n_cap : 0.0f;
 }
 
 // The same r_j from stored cosines (the normaliser Gram's output, the upper
@@ -115,16 +129,18 @@ int launch_capacity(const void* feats, int dtype, const float* inv, const float*
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
                     const DevParams& P, int64_t B, int64_t N, int64_t D, float* r, float* v,
                     float* v_out, cudaStream_t s, const float* cos, int64_t ldc) {
-  dim3 grid((unsigned)((N + 7) / 8), (unsigned)B);
+  // one block per token, a warp per neighbour (at most CAP_WARPS)
+  const dim3 grid((unsigned)N, (unsigned)B);
+  const int warps = P.n_cap < 1 ? 1 : (P.n_cap < CAP_WARPS ? P.n_cap : CAP_WARPS);
   if (cos)
     k_capacity_r_cos<<<dim3((unsigned)((N + 255) / 256), (unsigned)B), 256, 0, s>>>(
         cos, ldc, pos, frame, norms, nbr, P, (int)N, r);
   else if (dtype == CP_BF16)
-    k_capacity_r<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)feats, inv, pos, frame,
-                                                      norms, nbr, P, (int)N, (int)D, r);
+    k_capacity_r<__nv_bfloat16><<<grid, 32 * warps, 0, s>>>(
+        (const __nv_bfloat16*)feats, inv, pos, frame, norms, nbr, P, (int)N, (int)D, r);
   else
-    k_capacity_r<float><<<grid, 256, 0, s>>>((const float*)feats, inv, pos, frame, norms, nbr, P,
-                                             (int)N, (int)D, r);
+    k_capacity_r<float><<<grid, 32 * warps, 0, s>>>((const float*)feats, inv, pos, frame, norms,
+                                                        nbr, P, (int)N, (int)D, r);
   int st = last_launch_status();
   if (st != CP_OK) return st;
   k_capacity_v<<<(unsigned)B, 1024, 0, s>>>(r, (int)N, P.cap_mode, v, v_out);

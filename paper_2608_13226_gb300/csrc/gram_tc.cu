@@ -752,12 +752,18 @@ __global__ void __launch_bounds__(FP_THREADS, 4) k_fst_pair(
     const bool cols_in = jb + c4 + 3 < N;
     const size_t step16 = (size_t)16 * (size_t)ldc;
     float* up = cost + (sb + (size_t)(i0 + rl)) * (size_t)ldc + (jb + c4);
+    // every pass's cosines are loaded before the first store, so the four
+    // loads are in flight together (a store of pass p could otherwise alias
+    // the load of pass p + 1, which would wait for it)
+    float4 xs[FP_T / 16];
+#pragma unroll
+    for (int pass = 0; pass < FP_T / 16; ++pass)
+      xs[pass] = cols_ld ? __ldcs(reinterpret_cast<const float4*>(up + pass * step16))
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
     for (int pass = 0; pass < FP_T / 16; ++pass, up += step16) {
       const int r = pass * 16 + rl;
-      float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (cols_ld) x = __ldcs(reinterpret_cast<const float4*>(up));
-      const float c[4] = {x.x, x.y, x.z, x.w};
+      const float c[4] = {xs[pass].x, xs[pass].y, xs[pass].z, xs[pass].w};
       const float4 ti = s_ti[r];
       const float fi = s_fi[r];
       float o[4];

@@ -2,7 +2,7 @@
 profilers (ncu) and quick timing.
 
     python -m paper_2608_13226_gb300.profile_case --scene long_video --op select \
-        [--batch B] [--K K] [--g G] [--warmup W] [--repeat R]
+        [--batch B] [--K K] [--g G] [--norm-mode M] [--warmup W] [--repeat R]
 
 Prints one JSON line with the median CUDA-event time of the call.
 """
@@ -27,6 +27,8 @@ def main():
     ap.add_argument("--N", type=int, default=0, help="override the scene's token count")
     ap.add_argument("--K", type=int, default=0, help="0 = the workload's budget")
     ap.add_argument("--g", type=int, default=0)
+    ap.add_argument("--norm-mode", type=int, default=0, choices=(0, 1),
+                    help="feature normaliser: 0 min-max over all pairs, 1 bounded (d_f / 2)")
     ap.add_argument("--warmup", type=int, default=1)
     ap.add_argument("--repeat", type=int, default=3)
     a = ap.parse_args()
@@ -38,7 +40,7 @@ def main():
     pos = torch.from_numpy(np.stack([s["pos"] for s in sc])).cuda()
     fr = torch.from_numpy(np.stack([s["frame"] for s in sc])).cuda()
     K = a.K or cfg.K
-    prm = cp.Params(g=a.g)
+    prm = cp.Params(g=a.g, norm_mode=a.norm_mode)
     if a.op == "select":
         ws = cp.workspace(cp.CP_OP_SELECT, a.batch, cfg.N, cfg.D, K, cp._dtype(f), prm)
         run = lambda: cp.coverprune_select(f, pos, fr, K, prm, ws=ws)
