@@ -55,6 +55,7 @@ def test_defaults(lib):
     assert (p.alpha_f, p.alpha_x, p.alpha_tau) == (1.0, 1.0, 1.0)
     assert p.kappa == 10.0 and p.n_cap == 8 and p.g == 0 and p.capacity_mode == 0
     assert p.sgs_mode == 0
+    assert p.norm_mode == 0
     assert abs(p.voxel_m - 0.2) < 1e-7 and p.m0 == 0.0 and p.timeout_ms > 0
     py = cp.Params()
     for f in ("lambda_f", "kappa", "n_cap", "g", "voxel_m", "timeout_ms"):
@@ -128,6 +129,8 @@ def test_validation_rejects_before_launch(lib):
     assert _select(lib, params(capacity_mode=2)) == cp.CP_EINVAL
     assert _select(lib, params(timeout_ms=0.0)) == cp.CP_EINVAL
     assert _select(lib, params(sgs_mode=2)) == cp.CP_EINVAL
+    assert _select(lib, params(norm_mode=2)) == cp.CP_EINVAL
+    assert _select(lib, params(norm_mode=-1)) == cp.CP_EINVAL
     assert _select(lib, params(lambda_x=float("inf"))) == cp.CP_EINVAL
     # empty problems are no-ops
     assert _select(lib, p, B=0) == cp.CP_OK
