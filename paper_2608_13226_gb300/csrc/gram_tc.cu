@@ -29,8 +29,9 @@
 //               Chunks above the diagonal leave through a per-warp 32 x 32
 //               shared-memory transpose (the same 4 KB), so that each store
 //               instruction writes 4 rows x 128 contiguous bytes: whole L2
-//               lines, which L2 takes without reading DRAM first; their
-//               mirror images are column stores, one 128-byte line each
+//               lines, which L2 takes without reading DRAM first; chunks
+//               crossing the diagonal store their pairs j >= i element by
+//               element, chunks below it store nothing
 // Stage hand-offs use mbarriers (a stage's "empty" barrier counts the
 // commits of both CTAs' MMA threads, multicast); the accumulator hand-off
 // uses tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
