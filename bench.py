@@ -343,7 +343,7 @@ def run_ours(args, rank, world, local_rank, raw):
     sgs_bytes_per_step = cstats["cost_bytes_read"]
     sgs_launch_ms = sgs_ms / max(sgs_launches, 1)
     sgs_gbs = (sgs_bytes_per_step / launches_per_step) / (sgs_launch_ms / 1000.0) / 1e9
-    roofline_sgs = {"bound": "hbm", "kernel": "k_sgs_lazy<dense>", "achieved": round(sgs_gbs, 1),
+    roofline_sgs = {"bound": "hbm", "kernel": "k_sgs_lazy_cl", "achieved": round(sgs_gbs, 1),
                     "peak": hbm, "unit": "GB/s", "frac": round(sgs_gbs / hbm, 4),
                     "traffic": read_traffic("k_sgs_lazy", sgs_bytes_per_step // launches_per_step),
                     "peak_source": peak_kind,
@@ -418,7 +418,7 @@ def run_ours(args, rank, world, local_rank, raw):
     f_ms = fprof["sgs"][0] / max(fprof["sgs"][1], 1)
     f_bytes = fstats["cost_bytes_read"]
     f_gbs = f_bytes / (f_ms / 1000.0) / 1e9
-    sweep = {"bound": "hbm", "kernel": "k_sgs<dense>", "achieved": round(f_gbs, 1), "peak": hbm,
+    sweep = {"bound": "hbm", "kernel": "k_sgs<0>", "achieved": round(f_gbs, 1), "peak": hbm,
              "unit": "GB/s", "frac": round(f_gbs / hbm, 4),
              "traffic": read_traffic("k_sgs", f_bytes),
              "algorithmic_bytes_per_launch": f_bytes, "avg_launch_ms": round(f_ms, 3)}
