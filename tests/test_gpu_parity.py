@@ -276,6 +276,31 @@ def test_sgs_bf16_teacher_forced(orc, N, K, g, seed):
         assert float(host(sel["objective"])) == 0.0
 
 
+def test_short_clip_full_config(orc):
+    """The short-clip workload at its own size (N=4096, D=1280 bf16,
+    K=410): the whole cost matrix and capacity against the oracle, the
+    greedy teacher-forced on the GPU's own cost, and Lite."""
+    s = scene("short_clip", 0)
+    K = s["K"]
+    assert (s["feats"].shape, K) == ((4096, 1280), 410)
+    prm = cp.Params()
+    sel, cst = _select_case(orc, s, K, prm)
+    F = f64(s)
+    nm = orc.normalisers(F, s["pos"], s["frame"])
+    op = oracle_params(orc, prm)
+    assert_cost_close(host(cst["cost"]),
+                      orc.cost_matrix(F, s["pos"], s["frame"], op.weights, nm), "bf16")
+    _, vo = orc.capacity(F, s["pos"], s["frame"], op.weights, nm, prm.n_cap)
+    assert_capacity_close(host(cst["capacity"]), vo, "bf16")
+    div, _ = check_sgs_teacher_forced(orc, host(cst["cost"]).astype(np.float64),
+                                      host(cst["capacity"]).astype(np.float64),
+                                      host(sel["order"]), host(sel["gains"]),
+                                      float(host(sel["objective"])), 3.0)
+    near = _lite_check(orc, s, K, prm, "bf16")
+    print(f"short clip: teacher-forced near-tie picks {div}/{K}, Lite near-tie prototypes "
+          f"{near}/{K}")
+
+
 def test_sgs_closed_forms():
     # identical tokens: dense keeps 0..K-1; local keeps {0} + {g .. g+K-2}
     N, K, g = 50, 6, 5
