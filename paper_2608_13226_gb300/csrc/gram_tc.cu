@@ -10,18 +10,23 @@
 // (k_fst_pair, HBM-bound: each cosine read once, C(i, j) and C(j, i)
 // written), which also sums the greedy's first gains.
 //
-// Persistent clusters of two CTAs (one CTA per SM).  The two CTAs of a
-// cluster compute the row tiles 2p and 2p+1 of the same 256-column tile:
-// each loads its own 128x64 A box and one 128-row half of the shared
-// 256x64 B box, multicast to both CTAs, so a CTA fetches 32 KB from L2 per
-// 64-deep step instead of 48 (measured: the normaliser GEMM 0.88 -> 0.95 of
-// the bf16 peak without the cosine stores).  Each CTA has 10 warps:
+// Persistent CTA pairs (clusters of two CTAs, one CTA per SM) issuing the
+// pair MMA tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 16): a unit is
+// the 256 x 256 tile of row tiles 2p, 2p+1 and one 256-column tile.  Each
+// CTA loads only its own operands into its own shared memory: its 128 rows
+// of A (row tile 2p + rank) and its 128-row half of B, so a CTA fetches
+// 32 KB from L2 per 64-deep step instead of the 48 KB a single-CTA M = 128,
+// N = 256 tile needs; the pair instruction reads both CTAs' halves.  Row
+// tile 2p + rank's accumulator lands in that CTA's own TMEM.  Each CTA has
+// 10 warps:
 //   warp 0      TMA producer: 128x64 bf16 boxes, 128-byte swizzle, into a
-//               4-stage shared-memory ring (48 KB a stage); a stage is
-//               refilled once both CTAs' MMAs have released it
-//   warp 1      allocates 512 TMEM columns; lane 0 issues
-//               tcgen05.mma.cta_group::1.kind::f16 (M=128, N=256, K=16) into
-//               one of two 128x256 fp32 accumulators (double buffer)
+//               6-stage shared-memory ring (32 KB a stage); both CTAs'
+//               copies signal the leader CTA's (rank 0) "full" barrier
+//               (.cta_group::2 form), which expects both CTAs' bytes
+//   warp 1      allocates 512 TMEM columns (both CTAs, collectively); in the
+//               leader lane 0 issues the pair MMA into one of two 128x256
+//               fp32 accumulators per CTA (double buffer) and commits to
+//               the barriers of both CTAs
 //   warps 2..9  epilogue: warps w and w+4 share TMEM lane quadrant w%4 and
 //               split the 256 columns; tcgen05.ld 32 lanes x 32 columns at a
 //               time, cosines and their min/max in registers; the 32
@@ -31,13 +36,13 @@
 //               instruction writes 4 rows x 128 contiguous bytes: whole L2
 //               lines, which L2 takes without reading DRAM first; chunks
 //               crossing the diagonal store their pairs j >= i element by
-//               element, chunks below it store nothing
-// Stage hand-offs use mbarriers (a stage's "empty" barrier counts the
-// commits of both CTAs' MMA threads, multicast); the accumulator hand-off
-// uses tcgen05.commit -> mbarrier and back.  Every wait is bounded by the call's
-// time limit: on expiry the kernel records CP_ETIMEOUT, stops issuing work,
-// waits (bounded) for the copies and MMAs it already issued, frees its TMEM
-// and returns.
+//               element, chunks below it store nothing.  One lane a warp
+//               tells the leader that its accumulator is drained.
+// Stage hand-offs use mbarriers (a stage's "empty" barrier in each CTA gets
+// the leader's MMA commit); the accumulator hand-off uses tcgen05.commit ->
+// mbarrier and back.  Every wait is bounded by the call's time limit: on
+// expiry the kernel records CP_ETIMEOUT, stops issuing work, waits (bounded)
+// for the copies and MMAs it already issued, frees its TMEM and returns.
 #include <cuda.h>
 
 #include "common.cuh"
@@ -45,25 +50,27 @@
 namespace cp {
 namespace {
 
-constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 4;
+constexpr int TC_BM = 128, TC_BN = 256, TC_BK = 64, TC_STAGES = 6;
 constexpr int TC_EPI_WARPS = 8;                     // two per TMEM lane quadrant
 constexpr int TC_THREADS = 64 + 32 * TC_EPI_WARPS;  // producer, MMA, epilogue
-constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;  // 16 KB
-constexpr uint32_t TC_B_BYTES = TC_BN * TC_BK * 2;  // 32 KB
-constexpr uint32_t TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
+constexpr uint32_t TC_A_BYTES = TC_BM * TC_BK * 2;  // 16 KB: this CTA's 128 rows of A
+constexpr uint32_t TC_BH_BYTES = (TC_BN / 2) * TC_BK * 2;  // 16 KB: this CTA's half of B
+constexpr uint32_t TC_STAGE_BYTES = TC_A_BYTES + TC_BH_BYTES;
+constexpr uint32_t TC_PAIR_STAGE_BYTES = 2 * TC_STAGE_BYTES;  // what the leader's barrier expects
 constexpr uint32_t TC_TMEM_COLS = 512;              // 2 accumulators x 256 fp32 columns
 constexpr uint32_t TC_STG_FLOATS = 32 * 32;         // epilogue staging per warp (4 KB)
+constexpr uint32_t TC_EMPTY_ARRIVALS = 2 * TC_EPI_WARPS;  // one lane per epilogue warp, both CTAs
 constexpr size_t TC_SMEM = (size_t)TC_STAGES * TC_STAGE_BYTES +
                            (size_t)TC_EPI_WARPS * TC_STG_FLOATS * sizeof(float) +
                            1024;  // + alignment slack
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16,
-// both K-major, M = 128, N = 256.
+// both K-major, M = 256 (the CTA pair: 128 rows in each), N = 256.
 constexpr uint32_t kIdesc = (1u << 4)              // D format: f32
                             | (1u << 7)            // A format: bf16
                             | (1u << 10)           // B format: bf16
-                            | ((uint32_t)(TC_BN >> 3) << 17)   // N >> 3
-                            | ((uint32_t)(TC_BM >> 4) << 24);  // M >> 4
+                            | ((uint32_t)(TC_BN >> 3) << 17)        // N >> 3
+                            | ((uint32_t)((2 * TC_BM) >> 4) << 24);  // M >> 4
 
 struct TcArgs {
   const float4* tok;      // [B*N] (x, y, z, 1/||f||)
@@ -139,26 +146,28 @@ __device__ __forceinline__ uint64_t l2_policy_evict_first() {
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
-__device__ __forceinline__ void tma_load_3d(const CUtensorMap* map, uint64_t* bar, uint32_t dst,
-                                            int x, int y, int z, uint64_t policy) {
+// Cluster address of the same shared-memory object in the pair's CTA `rank`.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+  return r;
+}
+// A box into this CTA's shared memory at dst; the bytes are counted on the
+// mbarrier at cluster address bar_cl, which may lie in the peer CTA of the
+// pair (the .cta_group::2 form).
+__device__ __forceinline__ void tma_load_3d_pair(const CUtensorMap* map, uint32_t bar_cl,
+                                                 uint32_t dst, int x, int y, int z,
+                                                 uint64_t policy) {
   asm volatile(
       "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)),
-      "l"(policy)
+      ".cta_group::2.L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar_cl), "l"(policy)
       : "memory");
 }
-// The same box into the same shared-memory offset of every CTA in mask, each
-// CTA's mbarrier at that offset receiving the bytes.
-__device__ __forceinline__ void tma_load_3d_mc(const CUtensorMap* map, uint64_t* bar, uint32_t dst,
-                                               int x, int y, int z, uint16_t mask,
-                                               uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".multicast::cluster.L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6, %7;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "h"(mask),
-      "l"(policy)
-      : "memory");
+// Arrive (release at cluster scope) on the mbarrier at cluster address bar_cl.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cl) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cl)
+               : "memory");
 }
 __device__ __forceinline__ void st_f4_policy(float* p, const float4& v, uint64_t policy) {
   asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x),
@@ -186,22 +195,27 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
          | ((uint64_t)1 << 46)                     // descriptor version (fixed 0b001)
          | ((uint64_t)2 << 61);                    // swizzle mode: 128 B
 }
-__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
-                                          uint32_t accumulate) {
+// The pair MMA: D[256 x 256] (+)= A B^T, A's rows 0..127 from the leader's
+// shared memory and 128..255 from the peer's, B's columns 0..127 from the
+// leader's and 128..255 from the peer's (both at the same offsets); each
+// CTA's TMEM at tmem_d receives its own 128 rows.  Issued by one thread of
+// the leader CTA.
+__device__ __forceinline__ void umma_bf16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                               uint32_t accumulate) {
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
       "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
       : "memory");
 }
-// Arrive on the mbarrier at bar's offset in every CTA of mask once the MMAs
-// issued so far have completed.
-__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
+// Arrive on the mbarrier at bar's offset in both CTAs of the pair once the
+// pair MMAs issued so far have completed (an mbarrier signal, not a copy).
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
   asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
       " [%0], %1;" ::"r"(smem_u32(bar)),
-      "h"(mask)
+      "h"((uint16_t)0x3)
       : "memory");
 }
 __device__ __forceinline__ void cluster_sync_all() {
@@ -212,12 +226,6 @@ __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
   return r;
-}
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bar))
-      : "memory");
 }
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
@@ -288,29 +296,28 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t smem_base = (smem_u32(smem_raw) + 1023u) & ~1023u;  // 1024-B aligned ring
-  const int cr = (int)cluster_rank();                 // this CTA's row tile in the pair
+  const int cr = (int)cluster_rank();  // 0: the leader (issues the MMAs); 1: its peer
   const int cid = (int)(blockIdx.x >> 1), ncl = (int)(gridDim.x >> 1);
-  const uint16_t both = 0x3;
 
   if (threadIdx.x == 0) {
     s_abort = 0;
     for (int s = 0; s < TC_STAGES; ++s) {
-      mbar_init(&full_bar[s], 1);   // producer's arrive + the TMA bytes
-      mbar_init(&empty_bar[s], 2);  // a tcgen05.commit from each CTA of the pair
+      mbar_init(&full_bar[s], 1);   // leader only: its producer's arrive + both CTAs' bytes
+      mbar_init(&empty_bar[s], 1);  // the leader's MMA commit
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&tfull_bar[i], 1);     // one tcgen05.commit
-      mbar_init(&tempty_bar[i], 32 * TC_EPI_WARPS);  // every epilogue thread
+      mbar_init(&tfull_bar[i], 1);                   // the leader's MMA commit
+      mbar_init(&tempty_bar[i], TC_EMPTY_ARRIVALS);  // leader only: every epilogue warp
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
   }
-  if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+  if (warp == 1) {  // one warp of each CTA, collectively for the pair
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                      smem_u32(&s_tmem_base)),
                  "r"(TC_TMEM_COLS)
                  : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
   __syncthreads();
@@ -324,7 +331,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const uint64_t keep = l2_policy_evict_last();
       int stage = 0;
       uint32_t phase = 0;
-      uint32_t pending = 0;        // stages holding a load not yet seen consumed
+      uint32_t pending = 0;        // (leader) stages holding a load not yet seen consumed
       uint32_t pend_parity = 0;    // parity of that load's full phase, per stage bit
       for (int p = cid; p < a.total_pairs && !s_abort; p += ncl) {
         int b, I, J;
@@ -333,11 +340,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
           pending &= ~(1u << stage);
           const uint32_t sa = smem_base + (uint32_t)stage * TC_STAGE_BYTES;
-          mbar_arrive_expect_tx(&full_bar[stage], TC_STAGE_BYTES);
-          tma_load_3d(&mapA, &full_bar[stage], sa, kb * TC_BK, I * TC_BM, b, keep);
-          // own half of B into both CTAs; the peer's half arrives too
-          tma_load_3d_mc(&mapA, &full_bar[stage], sa + TC_A_BYTES + (uint32_t)cr * TC_A_BYTES,
-                         kb * TC_BK, J * TC_BN + cr * TC_BM, b, both, keep);
+          const uint32_t fb = cluster_addr(&full_bar[stage], 0);  // the leader's barrier
+          if (cr == 0) mbar_arrive_expect_tx(&full_bar[stage], TC_PAIR_STAGE_BYTES);
+          // this CTA's 128 rows of A, and its 128-row half of the 256-row B tile
+          tma_load_3d_pair(&mapA, fb, sa, kb * TC_BK, I * TC_BM, b, keep);
+          tma_load_3d_pair(&mapA, fb, sa + TC_A_BYTES, kb * TC_BK, J * TC_BN + cr * TC_BM, b,
+                           keep);
           pending |= 1u << stage;
           pend_parity = (pend_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == TC_STAGES) {
@@ -347,15 +355,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
       }
       if (s_abort) {
-        // let the copies already issued land before the block exits
-        const uint64_t drain = globaltimer_ns() + 50000000ull;
-        for (int s = 0; s < TC_STAGES; ++s)
-          if (pending & (1u << s))
-            while (!mbar_test(&full_bar[s], (pend_parity >> s) & 1u) && globaltimer_ns() < drain) {
-            }
+        // let the copies already issued land before the block exits: the
+        // leader sees them on its own barrier (a phase completes once both
+        // CTAs' bytes are in); the peer's copies signal the leader, so the
+        // peer waits a fixed bounded time instead
+        const uint64_t drain = globaltimer_ns() + (cr == 0 ? 50000000ull : 2000000ull);
+        if (cr == 0) {
+          for (int s = 0; s < TC_STAGES; ++s)
+            if (pending & (1u << s))
+              while (!mbar_test(&full_bar[s], (pend_parity >> s) & 1u) &&
+                     globaltimer_ns() < drain) {
+              }
+        } else if (pending) {
+          while (globaltimer_ns() < drain) {
+          }
+        }
       } else {
-        // every stage released by both MMAs: the peer's last commits to this
-        // CTA's barriers have landed before the final cluster barrier
+        // every stage released by the leader's MMAs: its last commits to
+        // this CTA's barriers have landed before the final cluster barrier
         for (int i = 0; i < TC_STAGES; ++i) {
           if (!mbar_wait(&empty_bar[stage], phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
           if (++stage == TC_STAGES) {
@@ -366,8 +383,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       }
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // ------------------------------------------------------------ MMA issuer (leader)
+    if (lane == 0 && cr == 0) {
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -389,9 +406,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           const uint64_t adesc = sw128_desc(sa), bdesc = sw128_desc(sa + TC_A_BYTES);
 #pragma unroll
           for (int k = 0; k < TC_BK / 16; ++k)  // 32 bytes further along K per step
-            umma_bf16(tmem_d, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k),
-                      (kb > 0 || k > 0) ? 1u : 0u);
-          umma_commit_mc(&empty_bar[stage], both);  // frees the stage (in both CTAs)
+            umma_bf16_pair(tmem_d, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(2 * k),
+                           (kb > 0 || k > 0) ? 1u : 0u);
+          umma_commit_pair(&empty_bar[stage]);  // frees the stage in both CTAs
           last_commit = &empty_bar[stage];
           last_parity = phase;
           if (++stage == TC_STAGES) {
@@ -400,7 +417,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
         }
         if (!ok) break;
-        umma_commit(&tfull_bar[acc]);  // accumulator ready for the epilogue
+        umma_commit_pair(&tfull_bar[acc]);  // both CTAs' accumulators ready for their epilogues
         last_commit = &tfull_bar[acc];
         last_parity = acc_phase;
         if (++acc == 2) {
@@ -426,6 +443,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                  ew * TC_STG_FLOATS;               // this warp's 32 x 32 staging tile
     float* s_rn = stg;  // the chunk columns' 1/||f||
     const uint64_t stream_out = l2_policy_evict_first();
+    const uint32_t tempty_cl0 = cluster_addr(&tempty_bar[0], 0);  // the leader's barriers
+    const uint32_t tempty_cl1 = cluster_addr(&tempty_bar[1], 0);
     int acc = 0;
     uint32_t acc_phase = 0;
     float cmax = -INFINITY, cmin = INFINITY;
@@ -524,7 +543,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(&tempty_bar[acc]);  // accumulator free for the MMA warp
+      __syncwarp();  // every lane's TMEM loads of this accumulator are done
+      if (lane == 0) mbar_arrive_cluster(acc ? tempty_cl1 : tempty_cl0);  // free for the leader's MMAs
       if (++acc == 2) {
         acc = 0;
         acc_phase ^= 1u;
@@ -535,9 +555,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  cluster_sync_all();  // the leader's MMAs and both CTAs' TMEM reads are over
+  if (warp == 1) {     // one warp of each CTA, collectively for the pair
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
                  "r"(TC_TMEM_COLS)
                  : "memory");
   }
