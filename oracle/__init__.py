@@ -126,9 +126,14 @@ def _load():
         lib.orc_lite_groups.argtypes = [_I64, _I64, _P, _P, _P, _P]
         lib.orc_lite_select.argtypes = [_I64, _I64, _P, _P, _P, C.POINTER(_Weights),
                                         C.POINTER(_Norms), _P, _P, _P, _I64, _P, _P, _P]
+        lib.orc_sot_sinkhorn.argtypes = [_I64, _I64, _P, _P, _P, C.c_double, _I64, _P, _P, _P,
+                                         _P]
+        lib.orc_sgs_literal.argtypes = [_I64, _P, _P, _I64, _P, _I64, C.c_double, _I64, _P, _P,
+                                        _P, _P, _P, _P]
         for fn in ("orc_normalisers", "orc_normalisers_mode", "orc_cost_rows", "orc_cost_pairs", "orc_knn_others",
                    "orc_capacity", "orc_objective", "orc_sgs", "orc_morton",
-                   "orc_lite_groups", "orc_lite_select"):
+                   "orc_lite_groups", "orc_lite_select", "orc_sot_sinkhorn",
+                   "orc_sgs_literal"):
             getattr(lib, fn).restype = C.c_int
         _lib = lib
         return lib
@@ -242,8 +247,12 @@ def capacity(F, X, tau, w: Weights, nm: Norms, n: int, nbr=None, mode: int = 0):
 # --------------------------------------------------------------------------
 
 def _nbr_g(nbr_g, N, g):
-    if g <= 0 or g >= N or nbr_g is None:
+    """(neighbour lists [N, g-1] or None, g): g <= 0 or g >= N (or no lists
+    given) means every token; g = 1 means the token alone."""
+    if g <= 0 or g >= N or (nbr_g is None and g != 1):
         return None, N
+    if g == 1:
+        return None, 1
     return np.ascontiguousarray(np.asarray(nbr_g, dtype=np.int32)[:, :g - 1]), g
 
 
@@ -280,6 +289,49 @@ def sgs(Cm, v, K: int, M0: float, g: int = 0, nbr_g=None, forced=None) -> dict:
                            _ptr(res["picked_gain"]), _ptr(res["F_after"])), "sgs")
     res["kept"] = np.sort(res["order"])
     res["F"] = float(res["F_after"][-1]) if K > 0 else float(M0 * v.sum())
+    return res
+
+
+def sot_sinkhorn(Crows, u, v, eps: float, iters: int, g0=None) -> dict:
+    """Entropic semi-relaxed OT (Eq. srpot_sinkhorn) between the sources of
+    the rows of Crows [m, N] (masses u) and N targets (capacities v), by
+    `iters` dual block-coordinate iterations from target potentials g0
+    (zeros by default).  Returns f [m], g [N], colsum = P^T 1 [N], P [m, N]."""
+    Crows = np.ascontiguousarray(np.asarray(Crows, dtype=np.float64))
+    m, N = Crows.shape
+    u, v = _f64(u), _f64(v)
+    g = np.zeros(N) if g0 is None else np.array(g0, dtype=np.float64)
+    f = np.empty(max(m, 1))
+    col = np.empty(N)
+    P = np.empty((m, N))
+    _check(_load().orc_sot_sinkhorn(m, N, _ptr(Crows), _ptr(u), _ptr(v), float(eps), int(iters),
+                                    _ptr(f), _ptr(g), _ptr(col), _ptr(P)), "sot_sinkhorn")
+    return {"f": f[:m], "g": g, "colsum": col, "P": P}
+
+
+def sgs_literal(Cm, v, K: int, eps: float, iters: int, g: int = 0, nbr_g=None,
+                forced=None) -> dict:
+    """K steps of SGS as Eqs. greedy_flow / sgs_select print it: residual
+    capacity r = [v - P^T 1]_+ of the entropic semi-relaxed OT from the
+    selected tokens (mass 1/K each), next token = argmin over unselected t
+    of sum_{j in M_g(t)} r_j C(t, j) (lowest index on exact ties).
+
+    Returns order, best_idx, best_score, second, picked_score (per step) and
+    kept (ascending).  With ``forced`` the oracle adds forced[l] at step l
+    but still reports its own argmin."""
+    Cm = _f64(Cm)
+    v = _f64(v)
+    N = Cm.shape[0]
+    nb, g = _nbr_g(nbr_g, N, g)
+    fo = None if forced is None else np.ascontiguousarray(np.asarray(forced, dtype=np.int64))
+    res = {k: np.empty(K, dtype=np.int64) for k in ("order", "best_idx")}
+    res.update({k: np.empty(K, dtype=np.float64) for k in
+                ("best_score", "second", "picked_score")})
+    _check(_load().orc_sgs_literal(N, _ptr(Cm), _ptr(v), g, _ptr(nb), K, float(eps), int(iters),
+                                   _ptr(fo), _ptr(res["order"]), _ptr(res["best_idx"]),
+                                   _ptr(res["best_score"]), _ptr(res["second"]),
+                                   _ptr(res["picked_score"])), "sgs_literal")
+    res["kept"] = np.sort(res["order"])
     return res
 
 

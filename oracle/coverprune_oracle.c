@@ -369,7 +369,7 @@ int orc_capacity(int64_t N, int64_t D, const double* F, const float* X,
  * or NULL for g == N. */
 static int in_neighbourhood(int64_t t, int64_t j, int64_t g, int64_t N,
                             const int32_t* nbr_g) {
-  if (g >= N || nbr_g == NULL) return 1;
+  if (g >= N) return 1;
   if (j == t) return 1;
   for (int64_t q = 0; q < g - 1; ++q)
     if (nbr_g[t * (g - 1) + q] == j) return 1;
@@ -380,7 +380,7 @@ static int in_neighbourhood(int64_t t, int64_t j, int64_t g, int64_t N,
 static double sgs_gain(int64_t t, int64_t N, const double* C, const double* v,
                        const double* m, int64_t g, const int32_t* nbr_g) {
   double acc = 0.0;
-  if (g >= N || nbr_g == NULL) {
+  if (g >= N) {
     for (int64_t j = 0; j < N; ++j) {
       double d = m[j] - C[t * N + j];
       if (d > 0.0) acc += v[j] * d;
@@ -405,6 +405,7 @@ int orc_objective(int64_t N, const double* C, const double* v, int64_t g,
                   double* out) {
   if (N < 1 || nS < 0 || !C || !v || !out) return ORC_EINVAL;
   if (g <= 0) g = N;
+  if (g > 1 && g < N && !nbr_g) return ORC_EINVAL;  /* M_g(t) needs t's g-1 neighbours */
   double F = 0.0;
   for (int64_t j = 0; j < N; ++j) {
     double m = M0;
@@ -439,6 +440,7 @@ int orc_sgs(int64_t N, const double* C, const double* v, int64_t g,
             double* picked_gain, double* F_after) {
   if (N < 1 || K < 0 || K > N || !C || !v) return ORC_EINVAL;
   if (g <= 0 || g > N) g = N;
+  if (g > 1 && g < N && !nbr_g) return ORC_EINVAL;
   double* m = (double*)malloc(sizeof(double) * (size_t)N);
   double* gain = (double*)malloc(sizeof(double) * (size_t)N);
   char* chosen = (char*)calloc((size_t)N, 1);
@@ -622,4 +624,172 @@ int orc_lite_select(int64_t N, int64_t D, const double* F, const float* X,
   free(nrm);
   if (objective) *objective = total;
   return ORC_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* Literal SGS with an entropic semi-relaxed OT (Sec. 3.5 read word for */
+/* word: Eqs. srpot_sinkhorn, greedy_flow, sgs_select, sgs_update)      */
+/* ------------------------------------------------------------------ */
+
+/* log(sum_k exp(x_k)) by shifting with the largest term; -inf when every
+ * term is -inf (or n == 0). */
+static double log_sum_exp(const double* x, int64_t n) {
+  double mx = -INFINITY;
+  for (int64_t k = 0; k < n; ++k)
+    if (x[k] > mx) mx = x[k];
+  if (mx == -INFINITY) return -INFINITY;
+  double s = 0.0;
+  for (int64_t k = 0; k < n; ++k) s += exp(x[k] - mx);
+  return mx + log(s);
+}
+
+/* Entropic semi-relaxed OT of Eq. srpot_sinkhorn,
+ *   min_P <C, P> - eps H(P)  s.t.  P 1 = u,  P^T 1 <= v,
+ * between m sources (row i of C holds C(source i, target j), j < N) and N
+ * targets, by block coordinate ascent on its dual.  The plan is
+ * P_ij = exp((f_i + g_j - C_ij) / eps) with g <= 0; each iteration first
+ * maximises the dual over f (rows: P 1 = u),
+ *   f_i = eps log u_i - eps log sum_j exp((g_j - C_ij) / eps),
+ * then over g <= 0 (columns: the capacity cap; a column below its capacity
+ * keeps g_j = 0),
+ *   g_j = min(0, eps log v_j - eps log sum_i exp((f_i - C_ij) / eps))
+ * (g_j = -inf when v_j = 0).  g holds the starting point on entry (zeros
+ * for a cold start) and the result on exit; f gets the row potentials.
+ * colsum (may be NULL) gets P^T 1 of the final potentials; P (may be NULL)
+ * the plan, [m, N].  The loops are plain; no tolerance stops them early. */
+int orc_sot_sinkhorn(int64_t m, int64_t N, const double* C, const double* u, const double* v,
+                     double eps, int64_t iters, double* f, double* g, double* colsum,
+                     double* P) {
+  if (m < 0 || N < 1 || iters < 0 || !(eps > 0.0) || (m > 0 && (!C || !u || !f)) || !v || !g)
+    return ORC_EINVAL;
+  int64_t w = m > N ? m : N;
+  double* x = (double*)malloc(sizeof(double) * (size_t)(w > 0 ? w : 1));
+  if (!x) return ORC_ENOMEM;
+  for (int64_t it = 0; it < iters && m > 0; ++it) {
+    for (int64_t i = 0; i < m; ++i) {
+      for (int64_t j = 0; j < N; ++j) x[j] = (g[j] - C[i * N + j]) / eps;
+      f[i] = eps * log(u[i]) - eps * log_sum_exp(x, N);
+    }
+    for (int64_t j = 0; j < N; ++j) {
+      if (!(v[j] > 0.0)) {
+        g[j] = -INFINITY;
+        continue;
+      }
+      for (int64_t i = 0; i < m; ++i) x[i] = (f[i] - C[i * N + j]) / eps;
+      double gj = eps * log(v[j]) - eps * log_sum_exp(x, m);
+      g[j] = gj < 0.0 ? gj : 0.0;
+    }
+  }
+  for (int64_t j = 0; j < N; ++j) {
+    double s = 0.0;
+    for (int64_t i = 0; i < m; ++i) {
+      double p = exp((f[i] + g[j] - C[i * N + j]) / eps);
+      if (P) P[i * N + j] = p;
+      s += p;
+    }
+    if (colsum) colsum[j] = s;
+  }
+  free(x);
+  return ORC_OK;
+}
+
+/* K steps of SGS as Eqs. greedy_flow and sgs_select print it (reading A10
+ * of the design notes; the default hot path uses the coverage-gain reading
+ * R5 instead).  At step l the sources are the l selected tokens, each with
+ * mass 1/K; the plan P_l of the entropic semi-relaxed OT against the target
+ * capacity v (orc_sot_sinkhorn, `iters` iterations, the target potentials
+ * warm-started from step l-1, zeros at l = 1) gives the residual capacity
+ *   r_j = max(v_j - (P_l^T 1)_j, 0)      (r = v at l = 0),
+ * and the next token minimises the residual-weighted local cost
+ *   score(t) = sum_{j in M_g(t)} r_j C(t, j)
+ * over the unselected tokens (lowest index among exact equals).  C [N, N]
+ * row = source; g <= 0 or g >= N means M_g = all tokens, else nbr_g [N,
+ * g-1] lists t's nearest others.
+ *
+ * forced (may be NULL): step l adds forced[l] instead of the argmin while
+ * the outputs still report the oracle's own argmin.  Outputs per step
+ * (any may be NULL): order (token added), best_idx / best_score (the
+ * argmin and its score), second (the smallest score among the other
+ * candidates, +inf if none), picked_score (score of the token added). */
+int orc_sgs_literal(int64_t N, const double* C, const double* v, int64_t g,
+                    const int32_t* nbr_g, int64_t K, double eps, int64_t iters,
+                    const int64_t* forced, int64_t* order, int64_t* best_idx,
+                    double* best_score, double* second, double* picked_score) {
+  if (N < 1 || K < 0 || K > N || !C || !v || !(eps > 0.0) || iters < 0) return ORC_EINVAL;
+  if (g <= 0 || g > N) g = N;
+  if (g > 1 && g < N && !nbr_g) return ORC_EINVAL;
+  int64_t* sel = (int64_t*)malloc(sizeof(int64_t) * (size_t)(K > 0 ? K : 1));
+  double* rows = (double*)malloc(sizeof(double) * (size_t)(K > 0 ? K : 1) * (size_t)N);
+  double* u = (double*)malloc(sizeof(double) * (size_t)(K > 0 ? K : 1));
+  double* fpot = (double*)malloc(sizeof(double) * (size_t)(K > 0 ? K : 1));
+  double* gpot = (double*)calloc((size_t)N, sizeof(double));
+  double* col = (double*)malloc(sizeof(double) * (size_t)N);
+  double* r = (double*)malloc(sizeof(double) * (size_t)N);
+  double* score = (double*)malloc(sizeof(double) * (size_t)N);
+  char* chosen = (char*)calloc((size_t)N, 1);
+  int rc = ORC_OK;
+  if (!sel || !rows || !u || !fpot || !gpot || !col || !r || !score || !chosen) {
+    rc = ORC_ENOMEM;
+    goto done;
+  }
+  for (int64_t l = 0; l < K; ++l) {
+    /* Eq. greedy_flow: residual target capacity after the step-l plan */
+    if (l == 0) {
+      for (int64_t j = 0; j < N; ++j) r[j] = v[j];
+    } else {
+      for (int64_t i = 0; i < l; ++i) u[i] = 1.0 / (double)K;
+      rc = orc_sot_sinkhorn(l, N, rows, u, v, eps, iters, fpot, gpot, col, NULL);
+      if (rc != ORC_OK) break;
+      for (int64_t j = 0; j < N; ++j) {
+        double d = v[j] - col[j];
+        r[j] = d > 0.0 ? d : 0.0;
+      }
+    }
+    /* Eq. sgs_select */
+#pragma omp parallel for schedule(static)
+    for (int64_t t = 0; t < N; ++t) {
+      if (chosen[t]) {
+        score[t] = INFINITY;
+        continue;
+      }
+      double s = 0.0;
+      if (g >= N) {
+        for (int64_t j = 0; j < N; ++j) s += r[j] * C[t * N + j];
+      } else {
+        s += r[t] * C[t * N + t];
+        for (int64_t q = 0; q < g - 1; ++q) {
+          int64_t j = nbr_g[t * (g - 1) + q];
+          s += r[j] * C[t * N + j];
+        }
+      }
+      score[t] = s;
+    }
+    int64_t b = -1;
+    for (int64_t t = 0; t < N; ++t)
+      if (!chosen[t] && (b < 0 || score[t] < score[b])) b = t;
+    double sec = INFINITY;
+    for (int64_t t = 0; t < N; ++t)
+      if (!chosen[t] && t != b && score[t] < sec) sec = score[t];
+    int64_t pick = b;
+    if (forced) {
+      pick = forced[l];
+      if (pick < 0 || pick >= N || chosen[pick]) {
+        rc = ORC_EINVAL;
+        break;
+      }
+    }
+    if (best_idx) best_idx[l] = b;
+    if (best_score) best_score[l] = score[b];
+    if (second) second[l] = sec;
+    if (picked_score) picked_score[l] = score[pick];
+    if (order) order[l] = pick;
+    /* Eq. sgs_update */
+    chosen[pick] = 1;
+    sel[l] = pick;
+    memcpy(rows + l * N, C + pick * N, sizeof(double) * (size_t)N);
+  }
+done:
+  free(sel); free(rows); free(u); free(fpot); free(gpot); free(col); free(r); free(score);
+  free(chosen);
+  return rc;
 }

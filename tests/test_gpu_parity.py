@@ -8,8 +8,8 @@ import torch
 
 import paper_2608_13226_gb300 as cp
 from gpu_util import (assert_capacity_close, assert_cost_close, batch_to_dev,
-                      check_sgs_end_to_end, check_sgs_teacher_forced, oracle_params, scene,
-                      to_dev)
+                      check_lite_end_to_end, check_sgs_end_to_end, check_sgs_teacher_forced,
+                      measured_errors, oracle_params, scene, to_dev)
 
 pytestmark = pytest.mark.gpu
 
@@ -278,27 +278,37 @@ def test_sgs_bf16_teacher_forced(orc, N, K, g, seed):
 
 def test_short_clip_full_config(orc):
     """The short-clip workload at its own size (N=4096, D=1280 bf16,
-    K=410): the whole cost matrix and capacity against the oracle, the
-    greedy teacher-forced on the GPU's own cost, and Lite."""
+    K=410): the whole cost matrix and capacity against the oracle; the
+    greedy teacher-forced over every step on the GPU's own cost and end to
+    end against the oracle's greedy on its own cost; Lite teacher-forced on
+    the GPU's capacity and end to end against the oracle's Lite."""
     s = scene("short_clip", 0)
     K = s["K"]
     assert (s["feats"].shape, K) == ((4096, 1280), 410)
     prm = cp.Params()
     sel, cst = _select_case(orc, s, K, prm)
     F = f64(s)
-    nm = orc.normalisers(F, s["pos"], s["frame"])
     op = oracle_params(orc, prm)
-    assert_cost_close(host(cst["cost"]),
-                      orc.cost_matrix(F, s["pos"], s["frame"], op.weights, nm), "bf16")
-    _, vo = orc.capacity(F, s["pos"], s["frame"], op.weights, nm, prm.n_cap)
-    assert_capacity_close(host(cst["capacity"]), vo, "bf16")
+    ora = orc.select(F, s["pos"], s["frame"], K, op)
+    assert_cost_close(host(cst["cost"]), ora["C"], "bf16")
+    assert_capacity_close(host(cst["capacity"]), ora["v"], "bf16")
+    order, kept = host(sel["order"]), host(sel["kept"])
     div, _ = check_sgs_teacher_forced(orc, host(cst["cost"]).astype(np.float64),
                                       host(cst["capacity"]).astype(np.float64),
-                                      host(sel["order"]), host(sel["gains"]),
+                                      order, host(sel["gains"]),
                                       float(host(sel["objective"])), 3.0)
+    eps = measured_errors(host(cst["cost"]), ora["C"], host(cst["capacity"]), ora["v"])
+    first, jac = check_sgs_end_to_end(orc, ora, order, kept, 3.0, eps=eps)
     near = _lite_check(orc, s, K, prm, "bf16")
-    print(f"short clip: teacher-forced near-tie picks {div}/{K}, Lite near-tie prototypes "
-          f"{near}/{K}")
+    f, pos, fr = to_dev(s)
+    lt = cp.coverprune_lite_select(f, pos, fr, K, prm)
+    torch.cuda.synchronize()
+    ora_l = orc.lite(F, s["pos"], s["frame"], K, op)
+    moved, near_e = check_lite_end_to_end(orc, s, ora_l, host(lt["kept"]),
+                                          host(lt["group_start"]), op.weights)
+    print(f"short clip: teacher-forced near-tie picks {div}/{K}, end to end equal for "
+          f"{first}/{K} steps (Jaccard {jac:.3f}); Lite near-tie prototypes {near}/{K} forced, "
+          f"{near_e} end to end, moved group starts {moved}")
 
 
 def test_sgs_closed_forms():
@@ -442,10 +452,20 @@ def _lite_check(orc, s, K, prm, dtype):
 @pytest.mark.parametrize("name,N,D,K", [("tiny", 1024, 256, 102), ("long_video", 1500, 512, 150),
                                         ("short_clip", 333, 256, 100)])
 def test_lite_parity(orc, name, N, D, K):
+    """Teacher-forced on the GPU's capacity, then end to end against the
+    oracle's Lite on its own normalisers, capacity and groups."""
     s = scene(name, 0, N=N, D=D)
     dtype = s["dtype"]
     near = _lite_check(orc, s, K, cp.Params(), dtype)
-    print(f"lite {name}: near-tie prototype differences {near}/{K}")
+    f, pos, fr = to_dev(s)
+    lt = cp.coverprune_lite_select(f, pos, fr, K)
+    torch.cuda.synchronize()
+    op = oracle_params(orc, cp.Params())
+    ora = orc.lite(f64(s), s["pos"], s["frame"], K, op)
+    moved, near_e = check_lite_end_to_end(orc, s, ora, host(lt["kept"]), host(lt["group_start"]),
+                                          op.weights, dtype)
+    print(f"lite {name}: near-tie prototype differences {near}/{K} forced, {near_e} end to "
+          f"end, moved group starts {moved}")
 
 
 @pytest.mark.parametrize("name,N,D,K", [("tiny", 1024, 256, 102), ("long_video", 1500, 512, 150)])

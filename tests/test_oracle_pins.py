@@ -301,6 +301,57 @@ def test_greedy_exhaustive(orc, seed, g):
     assert len(set(res["order"].tolist())) == K
 
 
+@pytest.mark.parametrize("seed", range(6))
+@pytest.mark.parametrize("g", [0, 3])
+def test_greedy_forced_order(orc, seed, g):
+    """Teacher forcing (the GPU parity tests drive the oracle's greedy along
+    the GPU's picks): forcing the oracle's own order reproduces its unforced
+    run exactly; forcing any other legal order adds exactly those tokens,
+    records as picked gain the exact objective decrease of each forced
+    addition, and still reports at every step the brute-force best addition
+    (argmax of the decrease over the unselected tokens, lowest index on
+    ties) and the runner-up's decrease."""
+    rng = np.random.default_rng(100 + seed)
+    N = int(rng.integers(7, 11))
+    K = int(rng.integers(2, 6))
+    F, X, tau = rand_scene(rng, N)
+    w = orc.Weights()
+    nm = orc.normalisers(F, X, tau)
+    Cm = orc.cost_matrix(F, X, tau, w, nm)
+    _, v = orc.capacity(F, X, tau, w, nm, 2)
+    M0 = 3.0
+    nbr = orc.knn_others(X, g - 1) if g else None
+    own = orc.sgs(Cm, v, K, M0, g, nbr)
+    again = orc.sgs(Cm, v, K, M0, g, nbr, forced=own["order"])
+    for k in ("order", "best_idx", "best_gain", "second", "picked_gain", "F_after"):
+        np.testing.assert_array_equal(again[k], own[k], err_msg=k)
+    np.testing.assert_array_equal(own["order"], own["best_idx"])
+    obj = lambda S: orc.objective(Cm, v, S, M0, g, nbr)
+    for trial in range(3):
+        forced = rng.permutation(N)[:K]
+        res = orc.sgs(Cm, v, K, M0, g, nbr, forced=forced)
+        np.testing.assert_array_equal(res["order"], forced)
+        prev = M0 * v.sum()
+        for l in range(K):
+            S = list(forced[:l])
+            dec = np.array([prev - obj(S + [t]) if t not in S else -np.inf for t in range(N)])
+            best = int(np.argmax(dec))  # first maximum = lowest index on exact ties
+            assert res["best_idx"][l] == best
+            assert res["best_gain"][l] == pytest.approx(dec[best], abs=1e-12)
+            rest = np.delete(dec, best)
+            second = rest.max() if np.isfinite(rest).any() else -1.0
+            assert res["second"][l] == pytest.approx(second, abs=1e-12)
+            cur = obj(S + [int(forced[l])])
+            assert res["picked_gain"][l] == pytest.approx(prev - cur, abs=1e-12)
+            assert res["F_after"][l] == pytest.approx(cur, abs=1e-12)
+            prev = cur
+    # a repeated or out-of-range forced token is an error, not a silent pick
+    with pytest.raises(ValueError):
+        orc.sgs(Cm, v, 2, M0, g, nbr, forced=np.array([1, 1]))
+    with pytest.raises(ValueError):
+        orc.sgs(Cm, v, 1, M0, g, nbr, forced=np.array([N]))
+
+
 # --------------------------------------------------------------------------
 # Closed forms
 # --------------------------------------------------------------------------

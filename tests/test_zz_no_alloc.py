@@ -34,7 +34,10 @@ def _positions(seed, B, N):
     return torch.from_numpy(x).cuda()
 
 
-@pytest.mark.parametrize("case", [(11, 3, 1500, 20), (12, 1, 777, 63)])
+# k = 8: the workspace entry point takes its grid kernel (lists in registers)
+# and this one its brute-force kernel; k = 0: the scene diameter alone
+@pytest.mark.parametrize("case", [(11, 3, 1500, 20), (12, 1, 777, 63), (13, 2, 1500, 8),
+                                  (14, 2, 900, 0)])
 def test_noalloc_matches_workspace_entry_point_twice(case):
     seed, B, N, k = case
     for call in range(2):  # two calls in a row; the second one changes sizes and data
