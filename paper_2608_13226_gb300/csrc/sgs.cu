@@ -646,7 +646,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_local(
 // after which no block touches another's shared memory.
 // ---------------------------------------------------------------------------
 constexpr int QD_QUADS = LZ_WARPS / 4;
-constexpr int CL_MAX = 8;  // blocks per cluster (portable cluster size)
+constexpr int CL_MAX = 16;  // blocks per cluster (16: the non-portable maximum)
 
 __device__ __forceinline__ void quad_sync(int k) {
   asm volatile("bar.sync %0, 128;" ::"r"(1 + k) : "memory");
@@ -1085,10 +1085,11 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   hw_cluster_sync();  // nobody leaves while a peer may still write to its shared memory
 }
 
-// Blocks per scene for the cluster kernel: the largest power of two <= 8
-// such that every scene's cluster can be resident at once.
+// Blocks per scene for the cluster kernel: the largest power of two <= 16
+// such that every scene's cluster can be resident at once (16 only where
+// the device runs that many clusters of 16 at a time; checked at launch).
 static int cluster_size_for(int64_t B, int sm_count) {
-  int C = 8;
+  int C = CL_MAX;
   while (C > 1 && (int64_t)C * B > sm_count) C >>= 1;
   return C;
 }
@@ -1116,7 +1117,7 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
     a.N = (int)N;
     a.K = (int)K;
     a.C = C;
-    a.lgC = C >= 8 ? 3 : C >= 4 ? 2 : C >= 2 ? 1 : 0;
+    a.lgC = C >= 16 ? 4 : C >= 8 ? 3 : C >= 4 ? 2 : C >= 2 ? 1 : 0;
     a.NC = (int)((N + C - 1) / C);
     a.nwords = (a.NC + 31) / 32;
     const int nit_max = (int)(((ldc / 4 + 31) / 32 + 3) / 4);  // iterations per quarter
@@ -1147,9 +1148,14 @@ static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* 
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    if (C > 8 && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                     cudaSuccess) {
+      (void)cudaGetLastError();
+      continue;
+    }
     int clusters = 0;
     if (cudaOccupancyMaxActiveClusters(&clusters, (const void*)fn, &cfg) != cudaSuccess ||
-        clusters < 1) {
+        clusters < 1 || (C > 8 && clusters < B)) {
       (void)cudaGetLastError();
       continue;  // this cluster shape cannot be resident: try a smaller one
     }
