@@ -41,7 +41,6 @@ WORKLOAD = "batch32_long_video_full_sgs_15pct"
 SCENES, RETENTION = 32, 0.15
 SCENE_NAME = "long_video"
 LOCAL_G = 64  # local neighbourhood size of the local-SGS measurement
-STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output")
 
 
 def _gen(seed):
@@ -681,14 +680,20 @@ def measure_configs(args, dev, stream, sync, max_over_ranks, feats, pos, fr, wor
         runs = [("select", select_call, prm)] if name != "lite_long" else []
         if name == "long_video":
             runs.append(("select_local_g64", select_call, cp.Params(g=LOCAL_G)))
+        if name != "lite_long":  # the rule as Sec. 3.5 prints it (entropic OT residual)
+            runs.append(("select_literal", select_call, cp.Params(sgs_mode=2)))
         runs += [("lite", lite_call, prm), ("lite_bounded", lite_call, bounded)]
         for key, mk, pr in runs:
             call, ws = mk(f, p_, t_, K, pr)
-            ms, stages = latency_of(call, stream)
+            slow = key == "select_literal" and N > 4096
+            ms, stages = latency_of(call, stream, reps=2 if slow else 5, warmup=1 if slow else 2)
             check(ws, f"{name} {key}")
             r = {"latency_ms": round(ms, 3), "stages_ms": stages}
             if key.startswith("select"):
                 r.update(sgs_numbers(stages, K, None, hbm))
+            if key == "select_literal":
+                r.update({"sot_eps": pr.sot_eps, "sot_iters": pr.sot_iters,
+                          "rule": "Eqs. greedy_flow / sgs_select as printed (sgs_mode 2)"})
             out.setdefault(name, ent)[key] = r
             del ws
         del f, p_, t_
@@ -715,17 +720,21 @@ def measure_configs(args, dev, stream, sync, max_over_ranks, feats, pos, fr, wor
                             "full_sweep_floor_ms": round(full_sweep_ms, 1)},
                            **sgs_numbers(stages, K, cbytes, hbm))
         if abs(R - RETENTION) < 1e-9:
-            pl = cp.Params(g=LOCAL_G)
-            call, ws = select_call(feats, pos, fr, K, pl)
-            ms, stages, _ = timed_calls(call, args.steps, args.warmup, stream, sync)
-            check(ws, "batch local select")
-            gst = cp.coverprune_call_stats(ws)
-            ms = max_over_ranks(ms)
-            e["select_local_g64"] = dict({"g": LOCAL_G, "scenes_per_s": B * world / (ms / 1000.0),
-                                          "ms_per_step": round(ms, 3), "stages_ms": stages,
-                                          "gain_evaluations_per_step": gst["gain_evaluations"]},
-                                         **sgs_numbers(stages, K, None, hbm))
-            del ws
+            # local SGS: with the min-max normaliser (the all-pairs Gram runs
+            # for the feature range and stores every cosine), and with the
+            # bounded one (only the Morton tiles holding a neighbour pair)
+            for key, pl in (("select_local_g64", cp.Params(g=LOCAL_G)),
+                            ("select_local_g64_bounded", cp.Params(g=LOCAL_G, norm_mode=1))):
+                call, ws = select_call(feats, pos, fr, K, pl)
+                ms, stages, _ = timed_calls(call, args.steps, args.warmup, stream, sync)
+                check(ws, f"batch {key}")
+                gst = cp.coverprune_call_stats(ws)
+                ms = max_over_ranks(ms)
+                e[key] = dict({"g": LOCAL_G, "scenes_per_s": B * world / (ms / 1000.0),
+                               "ms_per_step": round(ms, 3), "stages_ms": stages,
+                               "gain_evaluations_per_step": gst["gain_evaluations"]},
+                              **sgs_numbers(stages, K, None, hbm))
+                del ws
         floor_ms = B * N * D * 2 / (hbm * 1e9) * 1e3  # one read of the features
         for key, pr in (("lite", prm), ("lite_bounded", bounded)):
             call, ws = lite_call(feats, pos, fr, K, pr)

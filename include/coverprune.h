@@ -103,12 +103,34 @@ typedef enum {
  *   timeout_ms                      limit of every device-side wait, after
  *                                   which the kernel records CP_ETIMEOUT and
  *                                   returns (> 0; default 2000)
- *   sgs_mode                        how SGS finds each step's winner, with
- *                                   identical results: 0 = lazy (a gain
- *                                   computed at an earlier step bounds the
- *                                   current one, so only candidates whose
- *                                   bound could still win are re-evaluated;
- *                                   default), 1 = every gain every step
+ *   sgs_mode                        how SGS finds each step's winner: 0 =
+ *                                   lazy (a gain computed at an earlier step
+ *                                   bounds the current one, so only
+ *                                   candidates whose bound could still win
+ *                                   are re-evaluated; default), 1 = every
+ *                                   gain every step (the same picks); 2 =
+ *                                   the rule as Sec. 3.5 prints it: at step
+ *                                   l the entropic semi-relaxed OT of Eq.
+ *                                   srpot_sinkhorn from the l selected
+ *                                   tokens (mass 1/K each) to the target
+ *                                   capacity v gives the residual
+ *                                   r = [v - P^T 1]_+ (Eq. greedy_flow) and
+ *                                   the next token minimises
+ *                                   sum_{j in M_g(t)} r_j C(t, j) (Eq.
+ *                                   sgs_select; lowest index on ties); a
+ *                                   different selection, which scores a
+ *                                   candidate whose neighbourhood is already
+ *                                   served as 0 and so picks beside the
+ *                                   selected tokens (the default reading
+ *                                   maximises the coverage gain instead)
+ *   sot_eps                         entropic weight eps of Eq. srpot_sinkhorn
+ *                                   for sgs_mode 2 (> 0, finite; default
+ *                                   0.05 -- the paper gives no value)
+ *   sot_iters                       Sinkhorn iterations per greedy step for
+ *                                   sgs_mode 2 (1..10000; default 20; the
+ *                                   target potentials carry over from the
+ *                                   previous step -- the paper gives no
+ *                                   iteration count)
  *   norm_mode                       feature normaliser of Eq. fst_cost: 0 =
  *                                   min-max of d_f over all ordered pairs of
  *                                   the scene (Sec. 3.3; default); 1 =
@@ -133,6 +155,8 @@ typedef struct {
   float timeout_ms;
   int32_t sgs_mode;
   int32_t norm_mode;
+  float sot_eps;
+  int32_t sot_iters;
 } cp_params;
 
 /* Fills *p with the defaults listed above.  Host only; p must not be NULL. */
@@ -314,7 +338,10 @@ int coverprune_barrier_selftest(int32_t n_blocks, int32_t expected, float timeou
  * CP_STAGE_GRAM (feature normaliser GEMM), CP_STAGE_COST (cost GEMM),
  * CP_STAGE_CAPACITY, CP_STAGE_SGS (greedy selection incl. local slab),
  * CP_STAGE_LITE_ORDER (Morton order and groups), CP_STAGE_LITE_PROTO
- * (prototypes), CP_STAGE_OUTPUT (sort of kept indices, gather).
+ * (prototypes), CP_STAGE_OUTPUT (sort of kept indices, gather),
+ * CP_STAGE_SLAB (local SGS with the bounded feature normaliser: the Morton
+ * tile pairs that hold a neighbour pair and their cosines, in place of the
+ * all-pairs Gram).
  * Host only; thread-safe.  Returns CP_OK or CP_ECUDA.
  */
 typedef enum {
@@ -326,7 +353,8 @@ typedef enum {
   CP_STAGE_LITE_ORDER = 5,
   CP_STAGE_LITE_PROTO = 6,
   CP_STAGE_OUTPUT = 7,
-  CP_STAGE_COUNT = 8
+  CP_STAGE_SLAB = 8,
+  CP_STAGE_COUNT = 9
 } cp_stage;
 int coverprune_profile_enable(int on);
 int coverprune_profile_read(double* ms, int64_t* launches, int n);

@@ -28,7 +28,8 @@ EXPORTS = ("cp_default_params", "coverprune_budget", "coverprune_workspace_size"
            "coverprune_gather", "coverprune_barrier_selftest", "coverprune_profile_enable",
            "coverprune_profile_read", "coverprune_last_error", "coverprune_call_stats",
            "coverprune_version")
-STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output")
+STAGES = ("prep", "gram", "cost", "capacity", "sgs", "lite_order", "lite_proto", "output",
+          "slab")
 
 
 class CoverPruneError(RuntimeError):
@@ -47,7 +48,8 @@ class _CpParams(C.Structure):
                 ("alpha_f", C.c_float), ("alpha_x", C.c_float), ("alpha_tau", C.c_float),
                 ("n_cap", C.c_int32), ("g", C.c_int32), ("capacity_mode", C.c_int32),
                 ("voxel_m", C.c_float), ("m0", C.c_float), ("timeout_ms", C.c_float),
-                ("sgs_mode", C.c_int32), ("norm_mode", C.c_int32)]
+                ("sgs_mode", C.c_int32), ("norm_mode", C.c_int32),
+                ("sot_eps", C.c_float), ("sot_iters", C.c_int32)]
 
 
 class _CallStats(C.Structure):
@@ -74,6 +76,8 @@ class Params:
     timeout_ms: float = 2000.0
     sgs_mode: int = 0
     norm_mode: int = 0
+    sot_eps: float = 0.05
+    sot_iters: int = 20
 
     def _c(self) -> _CpParams:
         p = _CpParams()

@@ -153,7 +153,9 @@ static int check_params(const cp_params* p) {
   if (!(isfinite(p->timeout_ms) && p->timeout_ms > 0.0f)) return CP_EINVAL;
   if (p->n_cap < 0 || p->g < 0) return CP_EINVAL;
   if (p->capacity_mode != 0 && p->capacity_mode != 1) return CP_EINVAL;
-  if (p->sgs_mode != 0 && p->sgs_mode != 1) return CP_EINVAL;
+  if (p->sgs_mode < 0 || p->sgs_mode > 2) return CP_EINVAL;
+  if (!(isfinite(p->sot_eps) && p->sot_eps > 0.0f)) return CP_EINVAL;
+  if (p->sot_iters < 1 || p->sot_iters > 10000) return CP_EINVAL;
   if (p->norm_mode != 0 && p->norm_mode != 1) return CP_EINVAL;
   return CP_OK;
 }
@@ -186,6 +188,8 @@ static DevParams dev_params(const cp_params* p, int64_t N) {
   d.cap_mode = p->capacity_mode;
   d.sgs_mode = p->sgs_mode;
   d.norm_mode = p->norm_mode;
+  d.sot_eps = p->sot_eps;
+  d.sot_iters = p->sot_iters;
   d.timeout_ns = (uint64_t)((double)p->timeout_ms * 1.0e6);
   return d;
 }
@@ -197,6 +201,8 @@ struct Plan {
   size_t hdr, counters, stats, norms, inv, tok, nbr, r, v;
   size_t grid_info, grid_start, grid_pts;         // neighbour grid (kk <= kKnnGridMax)
   size_t cost, slab, partials, order32, g0;       // select
+  size_t lit;                                     // literal SGS (sgs_mode 2) scratch
+  size_t lfeats, ltok, lperm, lpos, lflags, lunits, lnunits;  // local Morton tiles
   size_t rev_off, rev;                            // local SGS reverse neighbourhoods
   size_t perm, prefix, gs, proto, score;          // lite
   size_t total;
@@ -214,7 +220,16 @@ static size_t knn_ws_bytes(int64_t B, int64_t N) {
          align_up(sizeof(float4) * (size_t)B * (size_t)N);
 }
 
-static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d, Plan* pl) {
+// Local SGS with the bounded feature normaliser on bf16 features computes
+// only the Morton tiles that hold a neighbour pair (local_slab.cu), not the
+// all-pairs Gram.
+static bool local_tiles_path(int op, int dtype, int64_t N, const DevParams& d) {
+  return op == CP_OP_SELECT && dtype == CP_BF16 && d.g < N && d.norm_mode == 1 &&
+         d.sgs_mode != 2;
+}
+
+static void plan_ws(int op, int64_t B, int64_t N, int64_t D, int64_t K, int dtype,
+                    const DevParams& d, Plan* pl) {
   memset(pl, 0, sizeof(*pl));
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -240,10 +255,21 @@ static void plan_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d,
   pl->v = take(sizeof(float) * BN);
   if (op == CP_OP_SELECT) {
     pl->cost = take(sizeof(float) * BN * (size_t)pl->ldc);
-    if (d.g < N) {
+    if (d.sgs_mode == 2) pl->lit = take(sgs_literal_ws_bytes(B, N, K));
+    if (d.g < N && d.sgs_mode != 2) {
       pl->slab = take(sizeof(float) * BN * (size_t)d.g);
       pl->rev_off = take(sizeof(int32_t) * (BN + (size_t)B));
       pl->rev = take(sizeof(int32_t) * BN * (size_t)d.g);
+    }
+    if (local_tiles_path(op, dtype, N, d)) {
+      const size_t T = (size_t)local_tiles(N);
+      pl->lfeats = take(2 * BN * (size_t)D);
+      pl->ltok = take(sizeof(float4) * BN);
+      pl->lperm = take(sizeof(int32_t) * BN);
+      pl->lpos = take(sizeof(int32_t) * BN);
+      pl->lflags = take((size_t)B * T * T);
+      pl->lunits = take(sizeof(uint32_t) * (size_t)B * T * T);
+      pl->lnunits = take(sizeof(int));
     }
     pl->partials = take(sizeof(uint64_t) * (size_t)sgs_partials_count(B, N));
     pl->order32 = take(sizeof(int32_t) * (size_t)B * (size_t)K);
@@ -327,9 +353,9 @@ static int check_inputs(const void* feats, const float* pos, const int32_t* fram
   return CP_OK;
 }
 
-static int check_ws(int op, int64_t B, int64_t N, int64_t K, const DevParams& d, void* ws,
-                    size_t ws_bytes, Plan* pl) {
-  plan_ws(op, B, N, K, d, pl);
+static int check_ws(int op, int64_t B, int64_t N, int64_t D, int64_t K, int dtype,
+                    const DevParams& d, void* ws, size_t ws_bytes, Plan* pl) {
+  plan_ws(op, B, N, D, K, dtype, d, pl);
   if (!ws || !aligned(ws, 256) || ws_bytes < pl->total) return CP_EWORKSPACE;
   return CP_OK;
 }
@@ -355,6 +381,8 @@ void cp_default_params(cp_params* p) {
   p->timeout_ms = 2000.0f;
   p->sgs_mode = 0;
   p->norm_mode = 0;
+  p->sot_eps = 0.05f;
+  p->sot_iters = 20;
 }
 
 int64_t coverprune_budget(double R, int64_t N) {
@@ -397,7 +425,7 @@ int coverprune_workspace_size(int op, int64_t B, int64_t N, int64_t D, int64_t K
   DevParams d = dev_params(p, N);
   CP_TRY(check_limits(op, N, d));
   Plan pl;
-  plan_ws(op, B, N, op == CP_OP_COST ? 0 : K, d, &pl);
+  plan_ws(op, B, N, D, op == CP_OP_COST ? 0 : K, dtype, d, &pl);
   *bytes = pl.total;
   return CP_OK;
 }
@@ -438,7 +466,7 @@ int coverprune_cost(const void* feats, int dtype, const float* pos, const int32_
   DevParams d = dev_params(p, N);
   CP_TRY(check_limits(CP_OP_COST, N, d));
   Plan pl;
-  CP_TRY(check_ws(CP_OP_COST, B, N, 0, d, ws, ws_bytes, &pl));
+  CP_TRY(check_ws(CP_OP_COST, B, N, D, 0, dtype, d, ws, ws_bytes, &pl));
   cudaStream_t s = (cudaStream_t)stream;
   // bf16: the normaliser pass stores the cosines into the output (the
   // capacity reads its pairs there), then one elementwise pass turns them
@@ -478,30 +506,52 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
   DevParams d = dev_params(p, N);
   CP_TRY(check_limits(CP_OP_SELECT, N, d));
   Plan pl;
-  CP_TRY(check_ws(CP_OP_SELECT, B, N, K, d, ws, ws_bytes, &pl));
+  CP_TRY(check_ws(CP_OP_SELECT, B, N, D, K, dtype, d, ws, ws_bytes, &pl));
   cudaStream_t s = (cudaStream_t)stream;
   int* status = at<int>(ws, pl.hdr);
   float* C = at<float>(ws, pl.cost);
-  CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, nullptr, s, C, pl.ldc));
+  // the all-pairs Gram stores every cosine into C for the cost pass; the
+  // local path with the bounded normaliser stores only the Morton tiles it
+  // needs (below), so the front runs no Gram for it
+  const bool tiles = local_tiles_path(CP_OP_SELECT, dtype, N, d);
+  CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, nullptr, s, tiles ? nullptr : C,
+                   pl.ldc));
   const SceneNorms* nm = at<SceneNorms>(ws, pl.norms);
   const float* inv = at<float>(ws, pl.inv);
   const int32_t* nbr = at<int32_t>(ws, pl.nbr);
   float* v = at<float>(ws, pl.v);
+  const int32_t* pos_of = nullptr;  // tiles: cos(t, j) at [min(pos)][max(pos)] of C
+  if (tiles) {
+    Stage st(CP_STAGE_SLAB, s);
+    int32_t* perm = at<int32_t>(ws, pl.lperm);
+    const int64_t T = local_tiles(N);
+    CP_TRY(launch_morton(pos, at<SceneStats>(ws, pl.stats), d, B, N, perm, s));
+    CP_TRY(launch_local_blocks(feats, at<float4>(ws, pl.tok), perm, nbr, d.kk, B, N, D,
+                               at<void>(ws, pl.lfeats), at<float4>(ws, pl.ltok),
+                               at<int32_t>(ws, pl.lpos), at<uint8_t>(ws, pl.lflags),
+                               at<uint32_t>(ws, pl.lunits), at<int>(ws, pl.lnunits), s));
+    CP_TRY(launch_gram_tiles(at<void>(ws, pl.lfeats), at<float4>(ws, pl.ltok), B, N, D,
+                             at<uint32_t>(ws, pl.lunits), at<int>(ws, pl.lnunits), B * T * T,
+                             status, d.timeout_ns, s, C, pl.ldc));
+    pos_of = at<int32_t>(ws, pl.lpos);
+  }
   {
     Stage st(CP_STAGE_CAPACITY, s);
     CP_TRY(launch_capacity(feats, dtype, inv, pos, frame, nm, nbr, d, B, N, D, at<float>(ws, pl.r),
-                           v, nullptr, s, dtype == CP_BF16 ? C : nullptr, pl.ldc));
+                           v, nullptr, s, dtype == CP_BF16 ? C : nullptr, pl.ldc, pos_of));
   }
   // the dense lazy selection starts from bounds the cost pass sums
   float* g0 = (dtype == CP_BF16 && d.g >= N && d.sgs_mode == 0) ? at<float>(ws, pl.g0) : nullptr;
   // local SGS reads only the N x g slab: for bf16 it comes straight from
-  // the stored cosines, and the dense cost is never formed
-  float* slab = d.g < N ? at<float>(ws, pl.slab) : nullptr;
+  // the stored cosines, and the dense cost is never formed (the literal rule
+  // transports from the selected tokens to every token, so it takes the
+  // dense cost whatever g is)
+  float* slab = (d.g < N && d.sgs_mode != 2) ? at<float>(ws, pl.slab) : nullptr;
   {
     Stage st(CP_STAGE_COST, s);
     if (dtype == CP_BF16 && slab)
       CP_TRY(launch_slab_cos(C, pl.ldc, nbr, at<float4>(ws, pl.tok), frame, nm, d, B, N, slab,
-                             s));
+                             s, pos_of));
     else if (dtype == CP_BF16)
       CP_TRY(launch_fst_apply(C, pl.ldc, B, N, at<float4>(ws, pl.tok), frame, nm, d, v, g0, s));
     else
@@ -512,10 +562,14 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
   {
     Stage st(CP_STAGE_SGS, s);
     if (slab && dtype != CP_BF16) CP_TRY(launch_slab(C, pl.ldc, nbr, d, B, N, slab, s));
-    CP_TRY(launch_sgs(C, pl.ldc, slab, nbr, v, d, B, N, K, order32, gains, objective,
-                      at<uint64_t>(ws, pl.partials), at<uint32_t>(ws, pl.counters), status, s,
-                      g0, slab ? at<int32_t>(ws, pl.rev_off) : nullptr,
-                      slab ? at<int32_t>(ws, pl.rev) : nullptr));
+    if (d.sgs_mode == 2)
+      CP_TRY(launch_sgs_literal(C, pl.ldc, nbr, v, d, B, N, K, order32, gains, objective,
+                                at<void>(ws, pl.lit), s));
+    else
+      CP_TRY(launch_sgs(C, pl.ldc, slab, nbr, v, d, B, N, K, order32, gains, objective,
+                        at<uint64_t>(ws, pl.partials), at<uint32_t>(ws, pl.counters), status, s,
+                        g0, slab ? at<int32_t>(ws, pl.rev_off) : nullptr,
+                        slab ? at<int32_t>(ws, pl.rev) : nullptr));
   }
   Stage st(CP_STAGE_OUTPUT, s);
   CP_TRY(launch_sort_kept(order32, B, K, kept, order, s));
@@ -538,7 +592,7 @@ int coverprune_lite_select(const void* feats, int dtype, const float* pos, const
   d.kk = d.n_cap;
   CP_TRY(check_limits(CP_OP_LITE, N, d));
   Plan pl;
-  CP_TRY(check_ws(CP_OP_LITE, B, N, K, d, ws, ws_bytes, &pl));
+  CP_TRY(check_ws(CP_OP_LITE, B, N, D, K, dtype, d, ws, ws_bytes, &pl));
   cudaStream_t s = (cudaStream_t)stream;
   CP_TRY(run_front(feats, dtype, pos, frame, B, N, D, d, pl, ws, nullptr, s));
   const SceneNorms* nm = at<SceneNorms>(ws, pl.norms);

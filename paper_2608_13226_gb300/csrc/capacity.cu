@@ -62,18 +62,21 @@ __global__ void __launch_bounds__(32 * CAP_WARPS) k_capacity_r(
   if (threadIdx.x == 0) r_all[(size_t)b * N + j] = P.n_cap > 0 ? acc / (float)P.n_cap : 0.0f;
 }
 
-// The same r_j from stored cosines (the normaliser Gram's output, the upper
-// triangle of [B][N][ldc]: cos(j, k) at [min(j, k)][max(j, k)]) in place of
-// the dot product, the rest identical.
+// The same r_j from stored cosines in place of the dot product, the rest
+// identical: the normaliser Gram's output, the upper triangle of
+// [B][N][ldc] (cos(j, k) at [min(j, k)][max(j, k)]); or, given pos_of, the
+// flagged Morton tiles of the local path (cos(j, k) at [min(pos)][max(pos)]).
 // One thread per token; its n gathers fall in one row, near its own index
 // (nearest neighbours sit in the same or adjacent frames).
 __global__ void __launch_bounds__(256) k_capacity_r_cos(
     const float* __restrict__ cos_all, int64_t ldc, const float* __restrict__ pos_all,
     const int32_t* __restrict__ frame_all, const SceneNorms* __restrict__ norms,
-    const int32_t* __restrict__ nbr_all, DevParams P, int N, float* __restrict__ r_all) {
+    const int32_t* __restrict__ nbr_all, DevParams P, int N, const int32_t* __restrict__ pos_of,
+    float* __restrict__ r_all) {
   const int j = blockIdx.x * 256 + threadIdx.x;
   const int b = blockIdx.y;
   if (j >= N) return;
+  const int32_t* po = pos_of ? pos_of + (size_t)b * N : nullptr;
   const float* crow = cos_all + ((size_t)b * N + j) * (size_t)ldc;
   const float* X = pos_all + (size_t)b * N * 3;
   const int32_t* TAU = frame_all + (size_t)b * N;
@@ -84,7 +87,13 @@ __global__ void __launch_bounds__(256) k_capacity_r_cos(
   float acc = 0.0f;
   for (int q = 0; q < P.n_cap; ++q) {
     const int k = nb[q];
-    const float cosv = k > j ? crow[k] : cos_all[((size_t)b * N + k) * (size_t)ldc + j];
+    float cosv;
+    if (po) {
+      const int a = po[j], c = po[k];
+      cosv = cos_all[((size_t)b * N + min(a, c)) * (size_t)ldc + max(a, c)];
+    } else {
+      cosv = k > j ? crow[k] : cos_all[((size_t)b * N + k) * (size_t)ldc + j];
+    }
     const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
     const float dx = sqrtf(sqdist_rn(xj, yj, zj, X[3 * k], X[3 * k + 1], X[3 * k + 2]));
     const float tx = (dx - nm.x_lo) * nm.x_rinv;
@@ -128,13 +137,14 @@ __global__ void __launch_bounds__(1024) k_capacity_v(const float* __restrict__ r
 int launch_capacity(const void* feats, int dtype, const float* inv, const float* pos,
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
                     const DevParams& P, int64_t B, int64_t N, int64_t D, float* r, float* v,
-                    float* v_out, cudaStream_t s, const float* cos, int64_t ldc) {
+                    float* v_out, cudaStream_t s, const float* cos, int64_t ldc,
+                    const int32_t* pos_of) {
   // one block per token, a warp per neighbour (at most CAP_WARPS)
   const dim3 grid((unsigned)N, (unsigned)B);
   const int warps = P.n_cap < 1 ? 1 : (P.n_cap < CAP_WARPS ? P.n_cap : CAP_WARPS);
   if (cos)
     k_capacity_r_cos<<<dim3((unsigned)((N + 255) / 256), (unsigned)B), 256, 0, s>>>(
-        cos, ldc, pos, frame, norms, nbr, P, (int)N, r);
+        cos, ldc, pos, frame, norms, nbr, P, (int)N, pos_of, r);
   else if (dtype == CP_BF16)
     k_capacity_r<__nv_bfloat16><<<grid, 32 * warps, 0, s>>>(
         (const __nv_bfloat16*)feats, inv, pos, frame, norms, nbr, P, (int)N, (int)D, r);

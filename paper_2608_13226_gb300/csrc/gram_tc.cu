@@ -82,6 +82,10 @@ struct TcArgs {
   int N, B, TI, TJ, num_kb;
   int pairs_per_scene, total_pairs;  // (row-tile pair, column tile) units
   uint64_t timeout_ns;
+  // tile-list mode (local SGS with the bounded normaliser): units[u] =
+  // (b << 16) | (P << 8) | J for u < *n_units, whole tiles stored, no min/max
+  const uint32_t* units;
+  const int* n_units;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -263,6 +267,13 @@ __device__ __forceinline__ void flush_minmax(SceneStats* st, float cmax, float c
 constexpr int TC_BAND = 8;
 __device__ __forceinline__ void unit_coords(const TcArgs& a, int p, int cr, int& b, int& I,
                                             int& J) {
+  if (a.units) {
+    const uint32_t u = __ldg(a.units + p);
+    b = (int)(u >> 16);
+    I = 2 * (int)((u >> 8) & 0xFFu) + cr;
+    J = (int)(u & 0xFFu);
+    return;
+  }
   b = p / a.pairs_per_scene;
   int r = p - b * a.pairs_per_scene;
   const int TP = (a.TI + 1) >> 1;  // == TJ
@@ -324,6 +335,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   tc_fence_after();
   cluster_sync_all();  // both CTAs' barriers exist before either signals the other
   const uint32_t tmem_base = s_tmem_base;
+  const int total = a.units ? *a.n_units : a.total_pairs;  // units of the whole grid
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -333,7 +345,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       uint32_t phase = 0;
       uint32_t pending = 0;        // (leader) stages holding a load not yet seen consumed
       uint32_t pend_parity = 0;    // parity of that load's full phase, per stage bit
-      for (int p = cid; p < a.total_pairs && !s_abort; p += ncl) {
+      for (int p = cid; p < total && !s_abort; p += ncl) {
         int b, I, J;
         unit_coords(a, p, cr, b, I, J);
         for (int kb = 0; kb < a.num_kb; ++kb) {
@@ -391,7 +403,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       uint32_t acc_phase = 0;
       uint64_t* last_commit = nullptr;
       uint32_t last_parity = 0;
-      for (int p = cid; p < a.total_pairs && !s_abort; p += ncl) {
+      for (int p = cid; p < total && !s_abort; p += ncl) {
         if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1u, &s_abort, a.timeout_ns, a.status)) break;
         tc_fence_after();
         const uint32_t tmem_d = tmem_base + (uint32_t)(acc * TC_BN);
@@ -449,7 +461,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     uint32_t acc_phase = 0;
     float cmax = -INFINITY, cmin = INFINITY;
     int cur_b = -1;
-    for (int p = cid; p < a.total_pairs; p += ncl) {
+    for (int p = cid; p < total; p += ncl) {
       // lane 0 waits, the warp follows it (keeps the warp converged for the
       // .sync.aligned TMEM loads below)
       int ok = 1;
@@ -460,7 +472,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       int b, I, J;
       unit_coords(a, p, cr, b, I, J);
       if (b != cur_b) {
-        if (cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
+        if (cur_b >= 0 && !a.units) flush_minmax(a.stats + cur_b, cmax, cmin);
         cur_b = b;
         cmax = -INFINITY;
         cmin = INFINITY;
@@ -502,7 +514,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         // only the upper triangle (j >= i) is stored: a chunk wholly above
         // the diagonal leaves through the transpose below, one crossing it
         // row by row; chunks below it store nothing
-        const int where = j0 >= r0 + 31 ? 1 : (j0 + 31 < r0 ? -1 : 0);
+        const int where = a.units ? 1 : (j0 >= r0 + 31 ? 1 : (j0 + 31 < r0 ? -1 : 0));
         if (where == 0 && row_ok) {
 #pragma unroll
           for (int e = 0; e < 32; ++e) {
@@ -550,7 +562,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         acc_phase ^= 1u;
       }
     }
-    if (cur_b >= 0) flush_minmax(a.stats + cur_b, cmax, cmin);
+    if (cur_b >= 0 && !a.units) flush_minmax(a.stats + cur_b, cmax, cmin);
   }
 
   tc_fence_before();
@@ -670,6 +682,57 @@ int launch_gram_minmax_tc(const void* feats, const float4* tok, int64_t B, int64
   const cudaError_t e = cudaLaunchKernelEx(&cfg, fn, mapA, a);
   note_launch();
   return cuda_status(e, "launch_gram_tc");
+}
+
+// The flagged tiles of the Morton-ordered features (local SGS with the
+// bounded normaliser): every unit of units[0 .. *n_units) in whole, stored at
+// its position coordinates in cos_out; at most max_units units.
+int launch_gram_tiles(const void* feats_m, const float4* tok_m, int64_t B, int64_t N, int64_t D,
+                      const uint32_t* units, const int* n_units, int64_t max_units, int* status,
+                      uint64_t timeout_ns, cudaStream_t s, float* cos_out, int64_t ldc) {
+  DeviceInfo di;
+  if (device_info(&di) != CP_OK) return CP_ECUDA;
+  alignas(64) CUtensorMap mapA;
+  CP_TRY_STATUS(make_feature_map(&mapA, feats_m, B, N, D, TC_BM));
+  TcArgs a{};
+  a.tok = tok_m;
+  a.cos_out = cos_out;
+  a.ldc = ldc;
+  a.vec_ok = (ldc % 4 == 0) && (reinterpret_cast<uintptr_t>(cos_out) % 16 == 0);
+  a.stats = nullptr;
+  a.status = status;
+  a.N = (int)N;
+  a.B = (int)B;
+  a.TI = (int)((N + TC_BM - 1) / TC_BM);
+  a.TJ = (int)((N + TC_BN - 1) / TC_BN);
+  a.num_kb = (int)((D + TC_BK - 1) / TC_BK);
+  a.pairs_per_scene = 0;
+  a.total_pairs = 0;
+  a.timeout_ns = timeout_ns;
+  a.units = units;
+  a.n_units = n_units;
+  if (max_units > INT_MAX) return CP_EUNSUPPORTED;
+  auto fn = k_gram_tc;
+  if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)TC_SMEM),
+                  "launch_gram_tiles: smem attribute") != CP_OK)
+    return CP_ECUDA;
+  const int64_t clusters = max_units < di.sm_count / 2 ? max_units : di.sm_count / 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(2 * (clusters > 0 ? clusters : 1)));
+  cfg.blockDim = dim3(TC_THREADS);
+  cfg.dynamicSmemBytes = TC_SMEM;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, fn, mapA, a);
+  note_launch();
+  return cuda_status(e, "launch_gram_tiles");
 }
 
 // ---------------------------------------------------------------------------
@@ -942,7 +1005,8 @@ __global__ void __launch_bounds__(256) k_slab_cos(const float* __restrict__ cos,
                                                   const float4* __restrict__ tok,
                                                   const int32_t* __restrict__ frame,
                                                   const SceneNorms* __restrict__ norms,
-                                                  DevParams P, float* __restrict__ slab) {
+                                                  DevParams P, const int32_t* __restrict__ pos_of,
+                                                  float* __restrict__ slab) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int b = blockIdx.y;
   if (i >= (int64_t)N * g) return;
@@ -951,7 +1015,15 @@ __global__ void __launch_bounds__(256) k_slab_cos(const float* __restrict__ cos,
   const int j = k == 0 ? t : __ldg(nbr + (sb + t) * kk + (k - 1));
   const FstConst kf = fst_const(norms[b], P);
   const float4 ti = __ldg(tok + sb + t), tj = __ldg(tok + sb + j);
-  const float c = __ldg(cos + (sb + min(t, j)) * (size_t)ldc + max(t, j));  // upper triangle
+  float c;
+  if (pos_of == nullptr)  // the upper triangle of the all-pairs Gram
+    c = __ldg(cos + (sb + min(t, j)) * (size_t)ldc + max(t, j));
+  else if (k == 0)        // cos(f, f) = 1 exactly, as the Gram's diagonal
+    c = ti.w > 0.0f ? 1.0f : 0.0f;
+  else {                  // the upper triangle of the flagged Morton tiles
+    const int pt = __ldg(pos_of + sb + t), pj = __ldg(pos_of + sb + j);
+    c = __ldg(cos + (sb + min(pt, pj)) * (size_t)ldc + max(pt, pj));
+  }
   slab[sb * g + i] = fst_cost_fold(kf, c, ti.x - tj.x, ti.y - tj.y, ti.z - tj.z,
                                    (float)__ldg(frame + sb + t), (float)__ldg(frame + sb + j));
 }
@@ -960,10 +1032,11 @@ __global__ void __launch_bounds__(256) k_slab_cos(const float* __restrict__ cos,
 
 int launch_slab_cos(const float* cos, int64_t ldc, const int32_t* nbr, const float4* tok,
                     const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
-                    int64_t N, float* slab, cudaStream_t s) {
+                    int64_t N, float* slab, cudaStream_t s, const int32_t* pos_of) {
   const int64_t n = N * P.g;
   dim3 grid((unsigned)((n + 255) / 256), (unsigned)B);
-  k_slab_cos<<<grid, 256, 0, s>>>(cos, ldc, (int)N, P.g, P.kk, nbr, tok, frame, norms, P, slab);
+  k_slab_cos<<<grid, 256, 0, s>>>(cos, ldc, (int)N, P.g, P.kk, nbr, tok, frame, norms, P, pos_of,
+                                  slab);
   return last_launch_status();
 }
 

@@ -20,8 +20,10 @@ struct DevParams {
   int g;       // SGS neighbourhood incl. the token itself; == N means all
   int kk;      // neighbours stored per token = max(n_cap, g-1) (g < N) or n_cap
   int cap_mode;
-  int sgs_mode;  // 0 = lazy evaluation of gains, 1 = every gain every step
+  int sgs_mode;  // 0 = lazy evaluation of gains, 1 = every gain every step, 2 = literal rule
   int norm_mode;  // feature normaliser: 0 = min-max over all pairs, 1 = d_f / 2
+  float sot_eps;  // literal rule: entropic weight of the semi-relaxed OT
+  int sot_iters;  // literal rule: Sinkhorn iterations per greedy step
   uint64_t timeout_ns;
 };
 
@@ -134,12 +136,27 @@ int launch_capacity(const void* feats, int dtype, const float* inv, const float*
                     const int32_t* frame, const SceneNorms* norms, const int32_t* nbr,
                     const DevParams& P, int64_t B, int64_t N, int64_t D, float* r, float* v,
                     float* v_out, cudaStream_t s, const float* cos = nullptr,
-                    int64_t ldc = 0);
+                    int64_t ldc = 0, const int32_t* pos_of = nullptr);
 // Local SGS, bf16 features: the same slab computed from the stored cosines
 // (cos [B][N][ldc], as the normaliser pass writes them), without a dense cost.
+// (pos_of given: cos(t, j) at [min(pos)][max(pos)] of the flagged Morton tiles).
 int launch_slab_cos(const float* cos, int64_t ldc, const int32_t* nbr, const float4* tok,
                     const int32_t* frame, const SceneNorms* norms, const DevParams& P, int64_t B,
-                    int64_t N, float* slab, cudaStream_t s);
+                    int64_t N, float* slab, cudaStream_t s, const int32_t* pos_of = nullptr);
+// Local SGS with the bounded normaliser, bf16 features: Morton-ordered
+// features and token records, each token's position, and the list of
+// 256 x 256 position tiles holding a neighbour pair (units (b << 16) |
+// (P << 8) | J, count in *n_units; at most B * T * T units, T = local_tiles(N)).
+int local_tiles(int64_t N);
+int launch_local_blocks(const void* feats, const float4* tok, const int32_t* perm,
+                        const int32_t* nbr, int kk, int64_t B, int64_t N, int64_t D,
+                        void* feats_m, float4* tok_m, int32_t* pos_of, uint8_t* flags,
+                        uint32_t* units, int* n_units, cudaStream_t s);
+// The listed tiles of the Gram of the Morton-ordered bf16 features, whole,
+// stored at their position coordinates in cos_out [B][N][ldc].
+int launch_gram_tiles(const void* feats_m, const float4* tok_m, int64_t B, int64_t N, int64_t D,
+                      const uint32_t* units, const int* n_units, int64_t max_units, int* status,
+                      uint64_t timeout_ns, cudaStream_t s, float* cos_out, int64_t ldc);
 // Local SGS: slab[b][t][k] = C(t, M_g(t)[k]) gathered from the dense cost.
 int launch_slab(const float* cost, int64_t ldc, const int32_t* nbr, const DevParams& P,
                 int64_t B, int64_t N, float* slab, cudaStream_t s);
@@ -154,6 +171,13 @@ int launch_sgs(const float* cost, int64_t ldc, const float* slab, const int32_t*
                int32_t* order32, float* gains, double* objective, uint64_t* partials,
                uint32_t* counters, int* status, cudaStream_t s, const float* g0 = nullptr,
                int32_t* rev_off = nullptr, int32_t* rev = nullptr);
+// K5 as Sec. 3.5 prints it (sgs_mode 2): entropic semi-relaxed OT residual
+// and the residual-weighted local cost; needs the dense cost [B][N][ldc]
+// and sgs_literal_ws_bytes(B, N, K) bytes of scratch (256-byte aligned).
+size_t sgs_literal_ws_bytes(int64_t B, int64_t N, int64_t K);
+int launch_sgs_literal(const float* cost, int64_t ldc, const int32_t* nbr, const float* v,
+                       const DevParams& P, int64_t B, int64_t N, int64_t K, int32_t* order32,
+                       float* gains, double* objective, void* scratch, cudaStream_t s);
 // Sort the B rows of K int32 indices ascending into int64 (and copy the
 // unsorted order out as int64 if order64 != NULL).
 int launch_sort_kept(const int32_t* idx32, int64_t B, int64_t K, int64_t* kept,

@@ -56,9 +56,11 @@ def test_defaults(lib):
     assert p.kappa == 10.0 and p.n_cap == 8 and p.g == 0 and p.capacity_mode == 0
     assert p.sgs_mode == 0
     assert p.norm_mode == 0
+    assert abs(p.sot_eps - 0.05) < 1e-7 and p.sot_iters == 20
     assert abs(p.voxel_m - 0.2) < 1e-7 and p.m0 == 0.0 and p.timeout_ms > 0
     py = cp.Params()
-    for f in ("lambda_f", "kappa", "n_cap", "g", "voxel_m", "timeout_ms"):
+    for f in ("lambda_f", "kappa", "n_cap", "g", "voxel_m", "timeout_ms", "sot_eps",
+              "sot_iters"):
         assert abs(getattr(py, f) - getattr(p, f)) < 1e-6
 
 
@@ -128,7 +130,12 @@ def test_validation_rejects_before_launch(lib):
     assert _select(lib, params(kappa=-1.0)) == cp.CP_EINVAL
     assert _select(lib, params(capacity_mode=2)) == cp.CP_EINVAL
     assert _select(lib, params(timeout_ms=0.0)) == cp.CP_EINVAL
-    assert _select(lib, params(sgs_mode=2)) == cp.CP_EINVAL
+    assert _select(lib, params(sgs_mode=3)) == cp.CP_EINVAL
+    assert _select(lib, params(sgs_mode=-1)) == cp.CP_EINVAL
+    assert _select(lib, params(sgs_mode=2, sot_eps=0.0)) == cp.CP_EINVAL
+    assert _select(lib, params(sgs_mode=2, sot_eps=float("nan"))) == cp.CP_EINVAL
+    assert _select(lib, params(sgs_mode=2, sot_iters=0)) == cp.CP_EINVAL
+    assert _select(lib, params(sgs_mode=2, sot_iters=10001)) == cp.CP_EINVAL
     assert _select(lib, params(norm_mode=2)) == cp.CP_EINVAL
     assert _select(lib, params(norm_mode=-1)) == cp.CP_EINVAL
     assert _select(lib, params(lambda_x=float("inf"))) == cp.CP_EINVAL
