@@ -38,6 +38,24 @@ template <> struct Vec16<__nv_bfloat16> {
 };
 
 // ---------------------------------------------------------------------------
+// Warp-level tensor-core tile (mma.sync m16n8k16, bf16 operands, fp32
+// accumulate): d += A B with A 16 x 16 (row-major; this lane holds rows
+// lane/4 and lane/4 + 8, columns 2 (lane % 4) + {0, 1} and + 8) and B 16 x 8
+// (column-major; this lane holds column lane/4, rows 2 (lane % 4) + {0, 1}
+// and + 8); d rows lane/4 and lane/4 + 8, columns 2 (lane % 4) + {0, 1}.
+// Each 32-bit operand register packs two consecutive bf16 of one row.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1,
+                                               uint32_t a2, uint32_t a3, uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// ---------------------------------------------------------------------------
 // Order-preserving float <-> uint32 keys (for atomicMin / atomicMax).
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t f2key(float f) {

@@ -191,30 +191,19 @@ int launch_groups(const float* v, const int32_t* perm, int64_t B, int64_t N, int
 
 // K8: prototype of each group (Eq. lite_select):
 //   s_q = argmin_{t in G_q} sum_{j in G_q} v_j C(t, j), lowest index on ties,
-// with C exactly as in the cost kernels.  One block per group; one warp per
-// candidate; the sum over targets runs in group order.
+// with C exactly as in the cost kernels.
+//
+// Scores of the members a = w, w + nwarps, ... of a group (warp w), each a
+// full-width dot product per pair; the sum over targets runs in group
+// order.  Keeps the warp's best (score, token).
 template <typename T>
-__global__ void __launch_bounds__(256) k_lite_proto(
-    const T* __restrict__ F_all, const float* __restrict__ inv_all, const float* __restrict__ pos_all,
-    const int32_t* __restrict__ frame_all, const SceneNorms* __restrict__ norms,
-    const float* __restrict__ v_all, const int32_t* __restrict__ perm_all,
-    const int32_t* __restrict__ gs_all, DevParams P, int N, int D, int K,
-    int32_t* __restrict__ proto, double* __restrict__ score) {
-  const int q = blockIdx.x, b = blockIdx.y;
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const T* F = F_all + (size_t)b * N * D;
-  const float* inv = inv_all + (size_t)b * N;
-  const float* X = pos_all + (size_t)b * N * 3;
-  const int32_t* TAU = frame_all + (size_t)b * N;
-  const float* v = v_all + (size_t)b * N;
-  const int32_t* gs = gs_all + (size_t)b * (K + 1);
-  const int32_t* mem = perm_all + (size_t)b * N + gs[q];
-  const int sz = gs[q + 1] - gs[q];
-  const SceneNorms nm = norms[b];
+__device__ __forceinline__ void lite_proto_simt(const T* F, const float* inv, const float* X,
+                                                const int32_t* TAU, const float* v,
+                                                const int32_t* mem, int sz, const SceneNorms& nm,
+                                                const DevParams& P, int D, int w, int lane,
+                                                int nwarps, float& best, int& best_t) {
   constexpr int V = Vec16<T>::n;
-  float best = INFINITY;
-  int best_t = INT32_MAX;
-  for (int a = w; a < sz; a += 8) {
+  for (int a = w; a < sz; a += nwarps) {
     const int t = mem[a];
     const T* ft = F + (size_t)t * D;
     const float xt = X[3 * t], yt = X[3 * t + 1], zt = X[3 * t + 2];
@@ -243,6 +232,27 @@ __global__ void __launch_bounds__(256) k_lite_proto(
       best_t = t;
     }
   }
+}
+
+// One block per group, one warp per candidate (fp32 features, and bf16
+// groups of more than LP_MAXG members).
+template <typename T>
+__global__ void __launch_bounds__(256) k_lite_proto(
+    const T* __restrict__ F_all, const float* __restrict__ inv_all, const float* __restrict__ pos_all,
+    const int32_t* __restrict__ frame_all, const SceneNorms* __restrict__ norms,
+    const float* __restrict__ v_all, const int32_t* __restrict__ perm_all,
+    const int32_t* __restrict__ gs_all, DevParams P, int N, int D, int K,
+    int32_t* __restrict__ proto, double* __restrict__ score) {
+  const int q = blockIdx.x, b = blockIdx.y;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int32_t* gs = gs_all + (size_t)b * (K + 1);
+  const int sz = gs[q + 1] - gs[q];
+  float best = INFINITY;
+  int best_t = INT32_MAX;
+  lite_proto_simt<T>(F_all + (size_t)b * N * D, inv_all + (size_t)b * N,
+                     pos_all + (size_t)b * N * 3, frame_all + (size_t)b * N,
+                     v_all + (size_t)b * N, perm_all + (size_t)b * N + gs[q], sz, norms[b], P, D,
+                     w, lane, 8, best, best_t);
   __shared__ float s_sc[8];
   __shared__ int s_t[8];
   if (lane == 0) {
@@ -252,6 +262,146 @@ __global__ void __launch_bounds__(256) k_lite_proto(
   __syncthreads();
   if (threadIdx.x == 0) {
     for (int i = 1; i < 8; ++i)
+      if (s_sc[i] < best || (s_sc[i] == best && s_t[i] < best_t)) {
+        best = s_sc[i];
+        best_t = s_t[i];
+      }
+    proto[(size_t)b * K + q] = best_t;
+    score[(size_t)b * K + q] = (double)best;
+  }
+}
+
+// bf16 features: the group's feature Gram on the tensor cores (mma.sync
+// m16n8k16, fp32 accumulate).  Members are taken in 16-row blocks and the
+// 16 x 16 tiles (bi <= bj) of X X^T are computed one after the other, the
+// feature width split over the block's 4 warps (warp w takes the 32-column
+// chunks w, w + 4, ...) and the four partial tiles added in warp order.  In
+// a chunk each lane loads 16 bytes of each of its rows (columns 8 (lane %
+// 4) ..): those 8 values feed two k16 steps, the columns' order along k
+// being the same for A and for B, so the dot products are unchanged.  A
+// block against itself reuses its A registers as B.  The tiles land, both
+// ways for bi < bj, in a shared-memory Gram, from which the scores read
+// every pair's dot product once.  Groups of more than LP_MAXG members
+// (rare: capacity-balanced groups are small) take the full-width loop.
+constexpr int LP_MAXG = 64, LP_WARPS = 4;
+__device__ __forceinline__ uint4 ld_row16(const __nv_bfloat16* row, int col, int D) {
+  return (row != nullptr && col < D) ? __ldg(reinterpret_cast<const uint4*>(row + col))
+                                     : make_uint4(0u, 0u, 0u, 0u);
+}
+__global__ void __launch_bounds__(32 * LP_WARPS) k_lite_proto_tc(
+    const __nv_bfloat16* __restrict__ F_all, const float* __restrict__ inv_all,
+    const float* __restrict__ pos_all, const int32_t* __restrict__ frame_all,
+    const SceneNorms* __restrict__ norms, const float* __restrict__ v_all,
+    const int32_t* __restrict__ perm_all, const int32_t* __restrict__ gs_all, DevParams P, int N,
+    int D, int K, int32_t* __restrict__ proto, double* __restrict__ score) {
+  __shared__ float s_dot[LP_MAXG][LP_MAXG + 1];
+  __shared__ float s_part[LP_WARPS][16][17];
+  __shared__ float s_inv[LP_MAXG], s_v[LP_MAXG], s_x[LP_MAXG][3];
+  __shared__ int s_mem[LP_MAXG], s_tau[LP_MAXG];
+  __shared__ float s_sc[LP_WARPS];
+  __shared__ int s_t[LP_WARPS];
+  const int q = blockIdx.x, b = blockIdx.y;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const __nv_bfloat16* F = F_all + (size_t)b * N * D;
+  const float* inv = inv_all + (size_t)b * N;
+  const float* X = pos_all + (size_t)b * N * 3;
+  const int32_t* TAU = frame_all + (size_t)b * N;
+  const float* v = v_all + (size_t)b * N;
+  const int32_t* gs = gs_all + (size_t)b * (K + 1);
+  const int32_t* mem = perm_all + (size_t)b * N + gs[q];
+  const int sz = gs[q + 1] - gs[q];
+  const SceneNorms nm = norms[b];
+  float best = INFINITY;
+  int best_t = INT32_MAX;
+  if (sz > LP_MAXG) {
+    lite_proto_simt<__nv_bfloat16>(F, inv, X, TAU, v, mem, sz, nm, P, D, w, lane, LP_WARPS, best,
+                                   best_t);
+  } else {
+    for (int a = threadIdx.x; a < sz; a += blockDim.x) {
+      const int t = mem[a];
+      s_mem[a] = t;
+      s_inv[a] = inv[t];
+      s_v[a] = v[t];
+      s_x[a][0] = X[3 * t];
+      s_x[a][1] = X[3 * t + 1];
+      s_x[a][2] = X[3 * t + 2];
+      s_tau[a] = TAU[t];
+    }
+    __syncthreads();
+    const int g = lane >> 2, tg = lane & 3;
+    const int nb = (sz + 15) >> 4;
+    for (int bi = 0; bi < nb; ++bi) {
+      for (int bj = bi; bj < nb; ++bj) {
+        const int ra0 = 16 * bi + g, ra1 = ra0 + 8, rb0 = 16 * bj + g, rb1 = rb0 + 8;
+        const __nv_bfloat16* pa0 = ra0 < sz ? F + (size_t)s_mem[ra0] * D : nullptr;
+        const __nv_bfloat16* pa1 = ra1 < sz ? F + (size_t)s_mem[ra1] * D : nullptr;
+        const __nv_bfloat16* pb0 = rb0 < sz ? F + (size_t)s_mem[rb0] * D : nullptr;
+        const __nv_bfloat16* pb1 = rb1 < sz ? F + (size_t)s_mem[rb1] * D : nullptr;
+        float d0[4] = {0.f, 0.f, 0.f, 0.f}, d1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 2
+        for (int c0 = 32 * w; c0 < D; c0 += 32 * LP_WARPS) {
+          const int col = c0 + 8 * tg;
+          const uint4 x0 = ld_row16(pa0, col, D), x1 = ld_row16(pa1, col, D);
+          uint4 y0 = x0, y1 = x1;  // bi == bj: B rows are A's
+          if (bi != bj) {
+            y0 = ld_row16(pb0, col, D);
+            y1 = ld_row16(pb1, col, D);
+          }
+          // k16 step over columns 8 tg + {0..3} of every lane, then + {4..7}
+          mma_bf16_16816(d0, x0.x, x1.x, x0.y, x1.y, y0.x, y0.y);
+          mma_bf16_16816(d1, x0.x, x1.x, x0.y, x1.y, y1.x, y1.y);
+          mma_bf16_16816(d0, x0.z, x1.z, x0.w, x1.w, y0.z, y0.w);
+          mma_bf16_16816(d1, x0.z, x1.z, x0.w, x1.w, y1.z, y1.w);
+        }
+        // d0: tile rows g (d0[0..1]) and g + 8 (d0[2..3]), columns 2 tg + {0, 1};
+        // d1: the same rows, columns 8 + 2 tg + {0, 1}
+        s_part[w][g][2 * tg] = d0[0];
+        s_part[w][g][2 * tg + 1] = d0[1];
+        s_part[w][g + 8][2 * tg] = d0[2];
+        s_part[w][g + 8][2 * tg + 1] = d0[3];
+        s_part[w][g][8 + 2 * tg] = d1[0];
+        s_part[w][g][9 + 2 * tg] = d1[1];
+        s_part[w][g + 8][8 + 2 * tg] = d1[2];
+        s_part[w][g + 8][9 + 2 * tg] = d1[3];
+        __syncthreads();
+        for (int e = threadIdx.x; e < 256; e += blockDim.x) {
+          const int r = e >> 4, c = e & 15;
+          const int rr = 16 * bi + r, cc = 16 * bj + c;
+          if (rr < sz && cc < sz) {
+            const float x = ((s_part[0][r][c] + s_part[1][r][c]) + s_part[2][r][c]) +
+                            s_part[3][r][c];
+            s_dot[rr][cc] = x;
+            if (bi != bj) s_dot[cc][rr] = x;
+          }
+        }
+        __syncthreads();  // s_part is reused by the next tile
+      }
+    }
+    for (int a = w; a < sz; a += LP_WARPS) {
+      const int t = s_mem[a];
+      const float inv_t = s_inv[a];
+      float sc = 0.0f;
+      for (int c = lane; c < sz; c += 32) {
+        float cosv = clamp_cos(s_dot[a][c] * inv_t * s_inv[c]);
+        if (c == a && inv_t > 0.0f) cosv = 1.0f;
+        const float d2 = sqdist_rn(s_x[a][0], s_x[a][1], s_x[a][2], s_x[c][0], s_x[c][1],
+                                   s_x[c][2]);
+        sc += s_v[c] * fst_cost_from(cosv, d2, s_tau[a], s_tau[c], nm, P);
+      }
+      sc = warp_sum(sc);
+      if (sc < best || (sc == best && t < best_t)) {
+        best = sc;
+        best_t = t;
+      }
+    }
+  }
+  if (lane == 0) {
+    s_sc[w] = best;
+    s_t[w] = best_t;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < LP_WARPS; ++i)
       if (s_sc[i] < best || (s_sc[i] == best && s_t[i] < best_t)) {
         best = s_sc[i];
         best_t = s_t[i];
@@ -285,9 +435,9 @@ int launch_lite_proto(const void* feats, int dtype, const float* inv, const floa
                       double* objective, cudaStream_t s) {
   dim3 grid((unsigned)K, (unsigned)B);
   if (dtype == CP_BF16)
-    k_lite_proto<__nv_bfloat16><<<grid, 256, 0, s>>>((const __nv_bfloat16*)feats, inv, pos, frame,
-                                                      norms, v, perm, gs, P, (int)N, (int)D, (int)K,
-                                                      proto, score);
+    k_lite_proto_tc<<<grid, 32 * LP_WARPS, 0, s>>>((const __nv_bfloat16*)feats, inv, pos, frame,
+                                                   norms, v, perm, gs, P, (int)N, (int)D, (int)K,
+                                                   proto, score);
   else
     k_lite_proto<float><<<grid, 256, 0, s>>>((const float*)feats, inv, pos, frame, norms, v, perm,
                                              gs, P, (int)N, (int)D, (int)K, proto, score);
