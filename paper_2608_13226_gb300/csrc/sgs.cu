@@ -841,15 +841,13 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     best = warp_max_u64(best);
     if (lane == 0) s_wq[w] = best;
   };
-  // quad leader: the quad's best key and whether it is exact (all_stale:
-  // at the start of a step after the first, without reading the bitmap,
-  // whose reset by other warps is not yet ordered before this read)
-  auto quad_best = [&](bool all_stale) -> unsigned long long {
+  // quad leader: the quad's best key and whether it is exact
+  auto quad_best = [&]() -> unsigned long long {
     unsigned long long kb = s_wq[4 * k];
     for (int i = 1; i < 4; ++i) kb = s_wq[4 * k + i] > kb ? s_wq[4 * k + i] : kb;
     const int bt = (int)(0xFFFFFFFFu - (uint32_t)(kb & 0xFFFFFFFFull)) >> lgC;
     s_qkey[k] = kb;
-    s_qfresh[k] = !all_stale && kb != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
+    s_qfresh[k] = kb != 0ull && ((fresh[bt >> 5] >> (bt & 31)) & 1u);
     return kb;
   };
 
@@ -859,12 +857,22 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
 
   for (int step = 0; step < a.K && ok; ++step) {
     // ---- step start: the quad bests into the first decision slot (the
-    // warp that held the last pick has rescanned; m is updated, fresh reset)
-    quad_sync(k);
-    if (q == 0 && lane == 0) {
-      const unsigned long long kb = quad_best(step > 0);
-      atomicMax(&s_G[slot], kb);
-      if (s_qfresh[k]) atomicMax(&s_BF[slot], kb);
+    // warp that held the last pick has rescanned; m is updated, and the
+    // bounds the pick may have changed are stale)
+    quad_sync(k);  // this quad's fresh bits and warp bests of the last step's end are settled
+    if (q == 0) {
+      unsigned long long kb = 0ull;
+      uint32_t fr = 0u;
+      if (lane == 0) {
+        kb = quad_best();
+        fr = s_qfresh[k];
+        atomicMax(&s_G[slot], kb);
+        if (fr) atomicMax(&s_BF[slot], kb);
+      }
+      kb = __shfl_sync(0xFFFFFFFFu, kb, 0);
+      fr = __shfl_sync(0xFFFFFFFFu, fr, 0);
+      if (fr && lane < a.C)  // an exact best from the start: lane r tells block r
+        red_dsmem_max_u64(map_rank(smem_addr(&s_hint), (uint32_t)lane), tag_key(kb, step));
     }
     if (threadIdx.x == 0) s_H[slot] = untag_key(ld_volatile_u64(&s_hint), step);
     __syncthreads();
@@ -929,7 +937,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
         quad_sync(k);
         if (w == 4 * k + ((tl >> 8) & 3)) warp_rescan();  // the warp holding t
         quad_sync(k);
-        if (q == 0 && lane == 0) (void)quad_best(false);
+        if (q == 0 && lane == 0) (void)quad_best();
       }
       if (q == 0 && lane == 0) {  // every quad into the next decision
         atomicMax(&s_G[slot], s_qkey[k]);
@@ -942,7 +950,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     // ---- phase 2: exchange the C results with their block masks.  Meanwhile
     // warp 1 of each quad prefetches into L2 the blocks of the quad's best
     // candidate, which the next step's first round will most likely
-    // re-evaluate (every bound goes stale with the pick)
+    // re-evaluate (most bounds go stale with the pick)
     const int par = step & 1;
     if (q == 1 && a.use_mask) {
       const unsigned long long kb = s_qkey[k];
@@ -1061,8 +1069,28 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
         }
       }
     }
-    // every bound goes stale; the warp that held the pick drops it
-    for (int i = threadIdx.x; i < a.nwords; i += LZ_THREADS) fresh[i] = 0u;
+    // A bound stays exact when its candidate had no positive term in any
+    // row block the pick lowers m on (the winner's mask WM): its terms, and
+    // so their rounded sum, are unchanged.  Its mask stays exact too (m is
+    // unchanged inside it).  Every other bound goes stale (all of them
+    // without masks); the warp that held the pick drops it.
+    // Each quad clears the bits of its own candidates (the ones its warps
+    // rescan), so a quad barrier orders them before the quad's next read.
+    if (a.use_mask) {
+      for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128) {
+        const uint32_t bit = 1u << (tl & 31);
+        if (fresh[tl >> 5] & bit) {  // only this thread changes this bit
+          const unsigned long long mk =
+              (unsigned long long)nzm[4 * tl] | ((unsigned long long)nzm[4 * tl + 1] << 16) |
+              ((unsigned long long)nzm[4 * tl + 2] << 32) |
+              ((unsigned long long)nzm[4 * tl + 3] << 48);
+          if (mk & WM) atomicAnd(&fresh[tl >> 5], ~bit);
+        }
+      }
+    } else {
+      for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128)
+        atomicAnd(&fresh[tl >> 5], ~(1u << (tl & 31)));
+    }
     if (own && w == 4 * (ptl & 7) + ((ptl >> 8) & 3)) {
       if (lane == 0) chosen[ptl >> 5] |= 1u << (ptl & 31);
       __syncwarp();

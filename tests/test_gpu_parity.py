@@ -35,7 +35,8 @@ def f64(s):
 # --------------------------------------------------------------------------
 
 @pytest.mark.parametrize("name,N,k", [("tiny", 1024, 8), ("short_clip", 4096, 63),
-                                      ("long_video", 1000, 17), ("tiny", 37, 36)])
+                                      ("long_video", 1000, 17), ("tiny", 37, 36),
+                                      ("long_video", 3000, 64), ("long_video", 2000, 65)])
 def test_knn_bit_exact(orc, name, N, k):
     s = scene(name, 1, N=N, D=64)
     _, pos, _ = to_dev(s)
@@ -561,6 +562,31 @@ def _lite_check(orc, s, K, prm, dtype):
             assert sc - score[q] <= 1e-5 * max(score[q], 1e-12), (q, t, proto[q], sc, score[q])
     assert abs(float(host(lt["objective"])) - total) <= 1e-4 * total + 1e-12
     return near
+
+
+@pytest.mark.parametrize("n_cap", [3, 8, 12])
+@pytest.mark.parametrize("N,D,seed", [(1001, 512, 6), (4100, 1280, 7)])
+def test_capacity_from_features(orc, n_cap, N, D, seed):
+    """The capacity computed from the bf16 features (Lite, and cost calls
+    without the cost) at ragged N and several neighbour counts, against the
+    oracle with the oracle's normalisers; Lite's capacity is the same (its
+    groups equal the oracle's grouping of this capacity)."""
+    s = scene("long_video", seed, N=N, D=D)
+    prm = cp.Params(n_cap=n_cap)
+    f, pos, fr = to_dev(s)
+    out = cp.coverprune_cost(f, pos, fr, prm, cost=False)
+    K = max(1, N // 10)
+    lt = cp.coverprune_lite_select(f, pos, fr, K, prm)
+    torch.cuda.synchronize()
+    op = oracle_params(orc, prm)
+    F = f64(s)
+    nm = orc.normalisers(F, s["pos"], s["frame"])
+    _, vo = orc.capacity(F, s["pos"], s["frame"], op.weights, nm, n_cap)
+    vg = host(out["capacity"])
+    assert_capacity_close(vg, vo, "bf16")
+    _, perm = orc.morton(s["pos"], prm.voxel_m)
+    b, _ = orc.lite_groups(vg, perm, K)
+    np.testing.assert_array_equal(host(lt["group_start"]), b)
 
 
 @pytest.mark.parametrize("name,N,D,K", [("tiny", 1024, 256, 102), ("long_video", 1500, 512, 150),
