@@ -2,7 +2,7 @@
 profilers (ncu) and quick timing.
 
     python -m paper_2608_13226_gb300.profile_case --scene long_video --op select \
-        [--batch B] [--K K] [--g G] [--norm-mode M] [--warmup W] [--repeat R]
+        [--batch B] [--K K] [--g G] [--norm-mode M] [--sgs-mode S] [--warmup W] [--repeat R]
 
 Prints one JSON line with the median CUDA-event time of the call.
 """
@@ -29,6 +29,8 @@ def main():
     ap.add_argument("--g", type=int, default=0)
     ap.add_argument("--norm-mode", type=int, default=0, choices=(0, 1),
                     help="feature normaliser: 0 min-max over all pairs, 1 bounded (d_f / 2)")
+    ap.add_argument("--sgs-mode", type=int, default=0, choices=(0, 1, 2),
+                    help="0 lazy, 1 every gain every step, 2 the rule as printed (entropic OT)")
     ap.add_argument("--warmup", type=int, default=1)
     ap.add_argument("--repeat", type=int, default=3)
     a = ap.parse_args()
@@ -40,7 +42,7 @@ def main():
     pos = torch.from_numpy(np.stack([s["pos"] for s in sc])).cuda()
     fr = torch.from_numpy(np.stack([s["frame"] for s in sc])).cuda()
     K = a.K or cfg.K
-    prm = cp.Params(g=a.g, norm_mode=a.norm_mode)
+    prm = cp.Params(g=a.g, norm_mode=a.norm_mode, sgs_mode=a.sgs_mode)
     if a.op == "select":
         ws = cp.workspace(cp.CP_OP_SELECT, a.batch, cfg.N, cfg.D, K, cp._dtype(f), prm)
         run = lambda: cp.coverprune_select(f, pos, fr, K, prm, ws=ws)
