@@ -645,7 +645,6 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_local(
 // return early: every block reaches the final hardware cluster barrier,
 // after which no block touches another's shared memory.
 // ---------------------------------------------------------------------------
-constexpr int QD_QUADS = LZ_WARPS / 4;
 constexpr int CL_MAX = 16;  // blocks per cluster (16: the non-portable maximum)
 
 __device__ __forceinline__ void quad_sync(int k) {
@@ -726,7 +725,15 @@ struct LzClArgs {
   uint32_t off_v, off_ub, off_chosen, off_fresh, off_nzm;  // dynamic smem offsets
 };
 
-__global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_constant__ LzClArgs a) {
+// WARPS warps a block (32: one block an SM; 16: two blocks an SM, of
+// different clusters, so one block runs while the other waits), in quads
+// of 4 warps.
+template <int WARPS>
+__global__ void __launch_bounds__(32 * WARPS, 1024 / (32 * WARPS))
+    k_sgs_lazy_cl(const __grid_constant__ LzClArgs a) {
+  constexpr int kThreads = 32 * WARPS, kQuads = WARPS / 4;
+  constexpr int kLQ = kQuads == 8 ? 3 : 2;  // log2(kQuads)
+  static_assert(kQuads == 8 || kQuads == 4, "4 or 8 quads");
   extern __shared__ __align__(16) unsigned char smem[];
   float* sm_m = reinterpret_cast<float*>(smem);                    // [ldc] coverage cost
   float* sm_v = reinterpret_cast<float*>(smem + a.off_v);          // [ldc] capacity
@@ -734,10 +741,10 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   uint32_t* chosen = reinterpret_cast<uint32_t*>(smem + a.off_chosen);  // [nwords]
   uint32_t* fresh = reinterpret_cast<uint32_t*>(smem + a.off_fresh);    // [nwords]
   uint16_t* nzm = reinterpret_cast<uint16_t*>(smem + a.off_nzm);   // [NC][4] if use_mask
-  __shared__ unsigned long long s_wq[LZ_WARPS];    // best key of each warp's candidates
-  __shared__ unsigned long long s_qkey[QD_QUADS];  // best key of each quad
-  __shared__ uint32_t s_qfresh[QD_QUADS];          // ... and whether it is exact
-  __shared__ float s_part[QD_QUADS][4];
+  __shared__ unsigned long long s_wq[WARPS];    // best key of each warp's candidates
+  __shared__ unsigned long long s_qkey[kQuads];  // best key of each quad
+  __shared__ uint32_t s_qfresh[kQuads];          // ... and whether it is exact
+  __shared__ float s_part[kQuads][4];
   __shared__ unsigned long long s_G[3], s_BF[3];   // block's largest key / largest exact
                                                    // key, one slot per round (mod 3)
   __shared__ unsigned long long s_hint;            // tagged; pushed by every block
@@ -755,19 +762,19 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int k = w >> 2, q = w & 3;
   // own index tl <-> candidate t = (tl << lgC) | crank; quad k scans the own
-  // indices k + 8 * (threadIdx.x & 127) + 1024 i, so warp 4 * (tl & 7) +
-  // ((tl >> 8) & 3) holds tl
+  // indices k + kQuads * (threadIdx.x & 127) + 128 kQuads i, so warp
+  // 4 * (tl & (kQuads - 1)) + ((tl >> (kLQ + 5)) & 3) holds tl
   const int nown = a.N > (int)crank ? (a.N - (int)crank + a.C - 1) >> lgC : 0;
   const float* Cb = a.cost + (size_t)(blockIdx.x >> lgC) * a.N * a.ldc;
 
   {
     const float* v = a.v + (size_t)(blockIdx.x >> lgC) * a.N;
-    for (int j = threadIdx.x; j < ncols; j += LZ_THREADS) {
+    for (int j = threadIdx.x; j < ncols; j += kThreads) {
       sm_m[j] = j < a.N ? a.m0 : 0.0f;
       sm_v[j] = j < a.N ? v[j] : 0.0f;
     }
   }
-  for (int i = threadIdx.x; i < a.nwords; i += LZ_THREADS) {
+  for (int i = threadIdx.x; i < a.nwords; i += kThreads) {
     chosen[i] = 0u;
     fresh[i] = a.g0 ? 0u : ~0u;  // step 0: exact gains from the sweep below, or bounds
   }
@@ -790,7 +797,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     // the two differ by a factor below 1 + 2^-9); scaled by 1 + 2^-8 and
     // rounded up they bound the gain, and are marked stale
     const float* g0 = a.g0 + (size_t)(blockIdx.x >> lgC) * a.g0_slots * a.N;
-    for (int tl = threadIdx.x; tl < nown; tl += LZ_THREADS) {
+    for (int tl = threadIdx.x; tl < nown; tl += kThreads) {
       const int t = (tl << lgC) | (int)crank;
       float sum = 0.0f;  // the slots in order; their loads issued together
 #pragma unroll 16
@@ -801,7 +808,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     }
   }
   // step 0 otherwise: every own candidate's gain exactly, one warp per row
-  for (int tl = a.g0 ? nown : w; tl < nown; tl += LZ_WARPS) {
+  for (int tl = a.g0 ? nown : w; tl < nown; tl += WARPS) {
     const float* crow = Cb + (size_t)((tl << lgC) | (int)crank) * a.ldc;
     float g0;
     if (a.use_mask) {
@@ -833,7 +840,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
   // the best key of this warp's remaining candidates, into s_wq[w]
   auto warp_rescan = [&]() {
     unsigned long long best = 0ull;
-    for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128)
+    for (int tl = k + kQuads * (threadIdx.x & 127); tl < nown; tl += kQuads * 128)
       if (!(chosen[tl >> 5] & (1u << (tl & 31)))) {
         const unsigned long long key = gain_key(ub[tl], (tl << lgC) | (int)crank);
         best = key > best ? key : best;
@@ -935,7 +942,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
             red_dsmem_max_u64(map_rank(smem_addr(&s_hint), (uint32_t)lane), tag_key(nk, step));
         }
         quad_sync(k);
-        if (w == 4 * k + ((tl >> 8) & 3)) warp_rescan();  // the warp holding t
+        if (w == 4 * k + ((tl >> (kLQ + 5)) & 3)) warp_rescan();  // the warp holding t
         quad_sync(k);
         if (q == 0 && lane == 0) (void)quad_best();
       }
@@ -1052,7 +1059,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
       const float4* row = reinterpret_cast<const float4*>(Cb + (size_t)pick * a.ldc);
       float4* m4 = reinterpret_cast<float4*>(sm_m);
       const int nq = ncols >> 2;
-      for (int bb = w; bb < 64; bb += LZ_WARPS) {
+      for (int bb = w; bb < 64; bb += WARPS) {
         if (!((WM >> bb) & 1ull)) continue;
         const int u0 = (bb & 15) << a.bit_shift, u1 = ((bb & 15) + 1) << a.bit_shift;
         for (int u = u0; u < u1; ++u) {
@@ -1077,7 +1084,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
     // Each quad clears the bits of its own candidates (the ones its warps
     // rescan), so a quad barrier orders them before the quad's next read.
     if (a.use_mask) {
-      for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128) {
+      for (int tl = k + kQuads * (threadIdx.x & 127); tl < nown; tl += kQuads * 128) {
         const uint32_t bit = 1u << (tl & 31);
         if (fresh[tl >> 5] & bit) {  // only this thread changes this bit
           const unsigned long long mk =
@@ -1088,10 +1095,10 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_lazy_cl(const __grid_cons
         }
       }
     } else {
-      for (int tl = k + QD_QUADS * (threadIdx.x & 127); tl < nown; tl += QD_QUADS * 128)
+      for (int tl = k + kQuads * (threadIdx.x & 127); tl < nown; tl += kQuads * 128)
         atomicAnd(&fresh[tl >> 5], ~(1u << (tl & 31)));
     }
-    if (own && w == 4 * (ptl & 7) + ((ptl >> 8) & 3)) {
+    if (own && w == 4 * (ptl & (kQuads - 1)) + ((ptl >> (kLQ + 5)) & 3)) {
       if (lane == 0) chosen[ptl >> 5] |= 1u << (ptl & 31);
       __syncwarp();
       warp_rescan();
@@ -1122,74 +1129,93 @@ static int cluster_size_for(int64_t B, int sm_count) {
   return C;
 }
 
+// One launch of the lazy kernel with WARPS warps a block on clusters of C
+// blocks.  Returns 1 (nothing launched) when that shape cannot be resident
+// -- every scene's cluster at once when all_resident -- else a status.
+template <int WARPS>
+static int lazy_launch_shape(LzClArgs a, int C, bool all_resident, int64_t B, int64_t N,
+                             int64_t ldc, const DeviceInfo& di, cudaStream_t s) {
+  auto fn = k_sgs_lazy_cl<WARPS>;
+  a.C = C;
+  a.lgC = C >= 16 ? 4 : C >= 8 ? 3 : C >= 4 ? 2 : C >= 2 ? 1 : 0;
+  a.NC = (int)((N + C - 1) / C);
+  a.nwords = (a.NC + 31) / 32;
+  const int nit_max = (int)(((ldc / 4 + 31) / 32 + 3) / 4);  // iterations per quarter
+  a.bit_shift = nit_max <= 16 ? 0 : 1;
+  a.off_v = (uint32_t)(sizeof(float) * ldc);
+  a.off_ub = (uint32_t)(sizeof(float) * 2 * ldc);
+  a.off_chosen = a.off_ub + (uint32_t)(sizeof(float) * a.NC);
+  a.off_fresh = a.off_chosen + (uint32_t)(sizeof(uint32_t) * a.nwords);
+  a.off_nzm = a.off_fresh + (uint32_t)(sizeof(uint32_t) * a.nwords);
+  const size_t smem_plain = a.off_nzm;
+  const size_t smem_mask = smem_plain + 4 * sizeof(uint16_t) * (size_t)a.NC;
+  // the block masks live in shared memory when they fit beside (m, v)
+  a.use_mask = smem_mask + 2048 <= (size_t)di.max_smem_optin ? 1 : 0;
+  const size_t smem = a.use_mask ? smem_mask : smem_plain;
+  if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem),
+                  "launch_sgs_lazy_cluster: smem attribute") != CP_OK)
+    return CP_ECUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(B * C));
+  cfg.blockDim = dim3(32 * WARPS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (C > 8 && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                   cudaSuccess) {
+    (void)cudaGetLastError();
+    return 1;
+  }
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, (const void*)fn, &cfg) != cudaSuccess ||
+      clusters < 1 || (all_resident && clusters < B)) {
+    (void)cudaGetLastError();
+    return 1;  // this cluster shape cannot be resident
+  }
+  cudaError_t e = cudaLaunchKernelEx(&cfg, fn, a);
+  note_launch();
+  return cuda_status(e, "launch_sgs_lazy_cluster");
+}
+
+// The cluster shape: C blocks of 32 warps, C the largest power of two <= 16
+// with every scene resident at once; where that C is below 16, clusters of
+// 2C blocks of 16 warps instead, two blocks an SM (from different
+// clusters), when every scene's cluster can be resident.
 static int sgs_lazy_cluster_launch(const float* cost, int64_t ldc, const float* v,
                                    const DevParams& P, int64_t B, int64_t N, int64_t K,
                                    int32_t* order32, float* gains, double* objective, int* status,
                                    cudaStream_t s, const float* g0) {
   DeviceInfo di;
   if (device_info(&di) != CP_OK) return CP_ECUDA;
-  auto fn = k_sgs_lazy_cl;
-  for (int C = cluster_size_for(B, di.sm_count); C >= 1; C >>= 1) {
-    LzClArgs a{};
-    a.cost = cost;
-    a.v = v;
-    a.g0 = g0;
-    a.g0_slots = fst_apply_slots(ldc);  // per column tile of the elementwise cost pass
-    a.order32 = order32;
-    a.gains = gains;
-    a.objective = objective;
-    a.status = status;
-    a.ldc = ldc;
-    a.timeout_ns = P.timeout_ns;
-    a.m0 = P.m0;
-    a.N = (int)N;
-    a.K = (int)K;
-    a.C = C;
-    a.lgC = C >= 16 ? 4 : C >= 8 ? 3 : C >= 4 ? 2 : C >= 2 ? 1 : 0;
-    a.NC = (int)((N + C - 1) / C);
-    a.nwords = (a.NC + 31) / 32;
-    const int nit_max = (int)(((ldc / 4 + 31) / 32 + 3) / 4);  // iterations per quarter
-    a.bit_shift = nit_max <= 16 ? 0 : 1;
-    a.off_v = (uint32_t)(sizeof(float) * ldc);
-    a.off_ub = (uint32_t)(sizeof(float) * 2 * ldc);
-    a.off_chosen = a.off_ub + (uint32_t)(sizeof(float) * a.NC);
-    a.off_fresh = a.off_chosen + (uint32_t)(sizeof(uint32_t) * a.nwords);
-    a.off_nzm = a.off_fresh + (uint32_t)(sizeof(uint32_t) * a.nwords);
-    const size_t smem_plain = a.off_nzm;
-    const size_t smem_mask = smem_plain + 4 * sizeof(uint16_t) * (size_t)a.NC;
-    // the block masks live in shared memory when they fit beside (m, v)
-    a.use_mask = smem_mask + 2048 <= (size_t)di.max_smem_optin ? 1 : 0;
-    const size_t smem = a.use_mask ? smem_mask : smem_plain;
-    if (cuda_status(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem),
-                    "launch_sgs_lazy_cluster: smem attribute") != CP_OK)
-      return CP_ECUDA;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(B * C));
-    cfg.blockDim = dim3(LZ_THREADS);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = (unsigned)C;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (C > 8 && cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-                     cudaSuccess) {
-      (void)cudaGetLastError();
-      continue;
-    }
-    int clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&clusters, (const void*)fn, &cfg) != cudaSuccess ||
-        clusters < 1 || (C > 8 && clusters < B)) {
-      (void)cudaGetLastError();
-      continue;  // this cluster shape cannot be resident: try a smaller one
-    }
-    cudaError_t e = cudaLaunchKernelEx(&cfg, fn, a);
-    note_launch();
-    return cuda_status(e, "launch_sgs_lazy_cluster");
+  LzClArgs a{};
+  a.cost = cost;
+  a.v = v;
+  a.g0 = g0;
+  a.g0_slots = fst_apply_slots(ldc);  // per column tile of the elementwise cost pass
+  a.order32 = order32;
+  a.gains = gains;
+  a.objective = objective;
+  a.status = status;
+  a.ldc = ldc;
+  a.timeout_ns = P.timeout_ns;
+  a.m0 = P.m0;
+  a.N = (int)N;
+  a.K = (int)K;
+  const int C32 = cluster_size_for(B, di.sm_count);
+  if (C32 < CL_MAX) {
+    const int st = lazy_launch_shape<16>(a, 2 * C32, true, B, N, ldc, di, s);
+    if (st != 1) return st;
+  }
+  for (int C = C32; C >= 1; C >>= 1) {
+    const int st = lazy_launch_shape<32>(a, C, C > 8, B, N, ldc, di, s);
+    if (st != 1) return st;
   }
   note_message("launch_sgs_lazy_cluster: no resident cluster shape");
   return CP_EUNSUPPORTED;

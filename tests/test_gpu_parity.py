@@ -483,7 +483,8 @@ def test_sgs_batch32_launch_shape(g):
                                              ("long_video", 3000, 256, 450, 0, 32),
                                              ("long_video", 2500, 256, 600, 64, 3),
                                              ("short_clip", 900, 128, 900, 12, 1),
-                                             ("long_video", 1200, 64, 300, 2, 2)])
+                                             ("long_video", 1200, 64, 300, 2, 2),
+                                             ("long_video", 1600, 128, 200, 0, 16)])
 def test_sgs_lazy_equals_full_sweep(name, N, D, K, g, B):
     """Lazy evaluation only skips candidates whose earlier (upper-bound) gain
     cannot win, so it must reproduce the full sweep bit for bit."""
