@@ -533,14 +533,17 @@ __global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos,
                                                   const int32_t* __restrict__ cell_start,
                                                   const float4* __restrict__ sorted,
                                                   int32_t* __restrict__ nbr) {
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  // thread jj takes the jj-th token in cell order: a warp's queries share
+  // their cells, so its lanes scan the same candidate cells together
+  const int jj = blockIdx.x * blockDim.x + threadIdx.x;
   const int b = blockIdx.y;
-  if (j >= N) return;
+  if (jj >= N) return;
   const GridInfo g = info[b];
-  const float* X = pos + (size_t)b * N * 3;
   const int32_t* cs = cell_start + (size_t)b * (gmax + 1);
   const float4* P = sorted + (size_t)b * N;
-  const float qx = X[3 * j], qy = X[3 * j + 1], qz = X[3 * j + 2];
+  const float4 qp = P[jj];
+  const int j = __float_as_int(qp.w);
+  const float qx = qp.x, qy = qp.y, qz = qp.z;
   const int cx = grid_coord(g, qx, 0), cy = grid_coord(g, qy, 1), cz = grid_coord(g, qz, 2);
   // only the first kk slots are used; the others stay at the smallest key
   // and never become the worst
@@ -605,25 +608,27 @@ __global__ void __launch_bounds__(128) k_knn_grid(const float* __restrict__ pos,
 }
 
 // More neighbours (8 < kk <= kKnnGridMax): the same shell search, one thread
-// per query, with the kk best keys in a max-heap in shared memory (slot i of
-// thread t at [i][t]: the threads of a warp touch distinct banks); the root
-// is the worst kept key.  A heapsort leaves them ascending at the end.
+// per query (queries in cell order), with the kk best keys in a max-heap in
+// shared memory (slot i of thread t at [i][t]: the threads of a warp touch
+// distinct banks); the root is the worst kept key.  A heapsort leaves them
+// ascending at the end.
 __global__ void __launch_bounds__(128) k_knn_grid_heap(const float* __restrict__ pos, int N, int kk,
                                                        int gmax, const GridInfo* __restrict__ info,
                                                        const int32_t* __restrict__ cell_start,
                                                        const float4* __restrict__ sorted,
                                                        int32_t* __restrict__ nbr) {
   extern __shared__ unsigned long long s_heap[];  // [kk][blockDim.x]
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  const int jj = blockIdx.x * blockDim.x + threadIdx.x;  // the jj-th token in cell order
   const int b = blockIdx.y;
-  if (j >= N) return;
+  if (jj >= N) return;
   const int T = blockDim.x;
   unsigned long long* H = s_heap + threadIdx.x;  // H[i * T] is slot i
   const GridInfo g = info[b];
-  const float* X = pos + (size_t)b * N * 3;
   const int32_t* cs = cell_start + (size_t)b * (gmax + 1);
   const float4* P = sorted + (size_t)b * N;
-  const float qx = X[3 * j], qy = X[3 * j + 1], qz = X[3 * j + 2];
+  const float4 qp = P[jj];
+  const int j = __float_as_int(qp.w);
+  const float qx = qp.x, qy = qp.y, qz = qp.z;
   const int cx = grid_coord(g, qx, 0), cy = grid_coord(g, qy, 1), cz = grid_coord(g, qz, 2);
   int cnt = 0;
   unsigned long long worst = ~0ull;  // the root once the heap is full

@@ -3,6 +3,7 @@ profilers (ncu) and quick timing.
 
     python -m paper_2608_13226_gb300.profile_case --scene long_video --op select \
         [--batch B] [--K K] [--g G] [--norm-mode M] [--sgs-mode S] [--warmup W] [--repeat R]
+        [--stages]
 
 Prints one JSON line with the median CUDA-event time of the call.
 """
@@ -33,6 +34,8 @@ def main():
                     help="0 lazy, 1 every gain every step, 2 the rule as printed (entropic OT)")
     ap.add_argument("--warmup", type=int, default=1)
     ap.add_argument("--repeat", type=int, default=3)
+    ap.add_argument("--stages", action="store_true",
+                    help="also report the per-stage split of the timed calls")
     a = ap.parse_args()
     cfg = scenes.config(a.scene, N=a.N) if a.N else scenes.CONFIGS[a.scene]
     sc = [scenes.make_scene(cfg, seed) for seed in range(a.batch)]
@@ -56,6 +59,9 @@ def main():
     for _ in range(a.warmup):
         run()
     torch.cuda.synchronize()
+    if a.stages:
+        cp.coverprune_profile_read()
+        cp.coverprune_profile_enable(True)
     times = []
     for _ in range(a.repeat):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -64,9 +70,16 @@ def main():
         e1.record()
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1))
+    stages = None
+    if a.stages:
+        cp.coverprune_profile_enable(False)
+        stages = {k: round(v[0] / a.repeat, 3) for k, v in cp.coverprune_profile_read().items()
+                  if v[0] > 0}
     st = cp.coverprune_check(ws)
     line = {"scene": a.scene, "op": a.op, "batch": a.batch, "N": cfg.N, "D": cfg.D, "K": K,
             "g": a.g, "ms_median": statistics.median(times), "status": cp.status_string(st)}
+    if stages is not None:
+        line["stages_ms"] = stages
     if a.op == "select":
         line["call_stats"] = cp.coverprune_call_stats(ws)
     print(json.dumps(line))

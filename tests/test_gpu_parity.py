@@ -36,7 +36,8 @@ def f64(s):
 
 @pytest.mark.parametrize("name,N,k", [("tiny", 1024, 8), ("short_clip", 4096, 63),
                                       ("long_video", 1000, 17), ("tiny", 37, 36),
-                                      ("long_video", 3000, 64), ("long_video", 2000, 65)])
+                                      ("long_video", 3000, 64), ("long_video", 2000, 65),
+                                      ("long_video", 8192, 8), ("long_video", 8192, 63)])
 def test_knn_bit_exact(orc, name, N, k):
     s = scene(name, 1, N=N, D=64)
     _, pos, _ = to_dev(s)
