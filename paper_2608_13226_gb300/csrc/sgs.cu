@@ -725,6 +725,39 @@ struct LzClArgs {
   uint32_t off_v, off_ub, off_chosen, off_fresh, off_nzm;  // dynamic smem offsets
 };
 
+// Every own unselected candidate's gain at the current m, warp w taking
+// own rows w, w + nwarps, ...: the quarter sums of its block mask folded as
+// combine_quarters does, so exactly a decision round's value; its mask is
+// renewed.  Kept out of line (called once a launch) so that the step loop
+// keeps its registers.
+__device__ __noinline__ void sweep_rows(const LzClArgs& a, const float* Cb, const float* sm_m,
+                                        const float* sm_v, float* ub, const uint32_t* chosen,
+                                        uint16_t* nzm, unsigned long long* s_stats, int nown,
+                                        uint32_t crank, int w, int nwarps, int lane) {
+  const int ncols = (int)a.ldc;
+  for (int tl = w; tl < nown; tl += nwarps) {
+    if (chosen[tl >> 5] & (1u << (tl & 31))) continue;
+    const float* crow = Cb + (size_t)((tl << a.lgC) | (int)crank) * a.ldc;
+    float g1 = 0.0f;
+    int nr_all = 0;
+#pragma unroll 1
+    for (int qq = 0; qq < 4; ++qq) {
+      uint32_t o;
+      int nr;
+      const float sq = quarter_gain_masked(crow, sm_m, sm_v, ncols, qq, lane, nzm[4 * tl + qq],
+                                           a.bit_shift, o, nr);
+      g1 = qq == 0 ? sq : __fadd_rn(g1, sq);
+      if (lane == 0) nzm[4 * tl + qq] = (uint16_t)o;
+      nr_all += nr;
+    }
+    if (lane == 0) {
+      ub[tl] = g1;
+      atomicAdd(&s_stats[0], 1ull);
+      atomicAdd(&s_stats[2], 512ull * (unsigned long long)nr_all);
+    }
+  }
+}
+
 // WARPS warps a block (32: one block an SM; 16: two blocks an SM, of
 // different clusters, so one block runs while the other waits), in quads
 // of 4 warps.
@@ -863,6 +896,20 @@ __global__ void __launch_bounds__(32 * WARPS, 1024 / (32 * WARPS))
   warp_rescan();  // step 0 starts from every warp's best
 
   for (int step = 0; step < a.K && ok; ++step) {
+    if (step == 1 && a.use_mask) {
+      // ---- step 1 as one sweep.  The first pick lowers m across the whole
+      // scene, so every bound left by step 0 is far above every gain of
+      // step 1 and the lazy rounds would evaluate all candidates anyway,
+      // one per quad and round.  Here each warp streams through its share
+      // of the block's rows instead, with no decision between rows: the
+      // same quarter sums in the same fold as a round's evaluation, so the
+      // same gains and masks.  Every bound is then exact.
+      __syncthreads();  // step 0's update of m and its chosen bit are done
+      sweep_rows(a, Cb, sm_m, sm_v, ub, chosen, nzm, s_stats, nown, crank, w, WARPS, lane);
+      for (int i = threadIdx.x; i < a.nwords; i += kThreads) fresh[i] = ~0u;
+      __syncthreads();
+      warp_rescan();
+    }
     // ---- step start: the quad bests into the first decision slot (the
     // warp that held the last pick has rescanned; m is updated, and the
     // bounds the pick may have changed are stale)
