@@ -11,6 +11,48 @@ namespace cp {
 // The dot products run over 16-byte feature vectors; the terms are summed in
 // neighbour order by one thread.
 constexpr int CAP_WARPS = 8;
+
+// acc + x . y over the 8 bf16 of each operand, element order lo, hi of each
+// 32-bit word in turn: fma.rn.f32.bf16 takes the bf16 operands as they are
+// (their product is exact in fp32) and rounds once, so each step equals
+// fmaf on the widened values and the sum is the same as widening first.
+__device__ __forceinline__ float dot8_bf16(const uint4 x, const uint4 y, float acc) {
+  asm("{\n\t.reg .b16 xl, xh, yl, yh;\n\t"
+      "mov.b32 {xl, xh}, %1;\n\tmov.b32 {yl, yh}, %5;\n\t"
+      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t"
+      "mov.b32 {xl, xh}, %2;\n\tmov.b32 {yl, yh}, %6;\n\t"
+      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t"
+      "mov.b32 {xl, xh}, %3;\n\tmov.b32 {yl, yh}, %7;\n\t"
+      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t"
+      "mov.b32 {xl, xh}, %4;\n\tmov.b32 {yl, yh}, %8;\n\t"
+      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t}"
+      : "+f"(acc)
+      : "r"(x.x), "r"(x.y), "r"(x.z), "r"(x.w), "r"(y.x), "r"(y.y), "r"(y.z), "r"(y.w));
+  return acc;
+}
+template <typename T>
+__device__ __forceinline__ float row_dot(const T* a, const T* b, int D, int lane) {
+  constexpr int V = Vec16<T>::n;
+  float dot = 0.0f;
+  for (int d = lane * V; d < D; d += 32 * V) {
+    float x[V], y[V];
+    Vec16<T>::load(a + d, x);
+    Vec16<T>::load(b + d, y);
+#pragma unroll
+    for (int i = 0; i < V; ++i) dot = fmaf(x[i], y[i], dot);
+  }
+  return dot;
+}
+template <>
+__device__ __forceinline__ float row_dot<__nv_bfloat16>(const __nv_bfloat16* a,
+                                                        const __nv_bfloat16* b, int D, int lane) {
+  float dot = 0.0f;
+  for (int d = lane * 8; d < D; d += 256)
+    dot = dot8_bf16(__ldg(reinterpret_cast<const uint4*>(a + d)),
+                    __ldg(reinterpret_cast<const uint4*>(b + d)), dot);
+  return dot;
+}
+
 template <typename T>
 __global__ void __launch_bounds__(32 * CAP_WARPS) k_capacity_r(
     const T* __restrict__ F_all, const float* __restrict__ inv_all, const float* __restrict__ pos_all,
@@ -28,7 +70,6 @@ __global__ void __launch_bounds__(32 * CAP_WARPS) k_capacity_r(
   const int32_t* TAU = frame_all + (size_t)b * N;
   const int32_t* nb = nbr_all + ((size_t)b * N + j) * P.kk;
   const SceneNorms nm = norms[b];
-  constexpr int V = Vec16<T>::n;
   const T* fj = F + (size_t)j * D;
   float acc = 0.0f;  // thread 0's running sum, in neighbour order
   for (int q0 = 0; q0 < P.n_cap; q0 += CHUNK) {
@@ -36,15 +77,7 @@ __global__ void __launch_bounds__(32 * CAP_WARPS) k_capacity_r(
     for (int qq = w; qq < qn; qq += nw) {
       const int k = __ldg(nb + q0 + qq);
       const T* fk = F + (size_t)k * D;
-      float dot = 0.0f;
-      for (int d = lane * V; d < D; d += 32 * V) {
-        float a[V], c[V];
-        Vec16<T>::load(fj + d, a);
-        Vec16<T>::load(fk + d, c);
-#pragma unroll
-        for (int i = 0; i < V; ++i) dot = fmaf(a[i], c[i], dot);
-      }
-      dot = warp_sum(dot);
+      const float dot = warp_sum(row_dot<T>(fj, fk, D, lane));
       const float cosv = clamp_cos(dot * inv[j] * inv[k]);
       const float tf = ((1.0f - cosv) - nm.f_lo) * nm.f_rinv;
       const float dx = sqrtf(sqdist_rn(X[3 * j], X[3 * j + 1], X[3 * j + 2], X[3 * k],
