@@ -1,6 +1,7 @@
 // K4: FST capacity (Sec. 3.4, Eqs. fst_capacity_score, fst_capacity) and the
 // cost slab of the local SGS neighbourhoods (Eq. local_neighbor).
 #include "common.cuh"
+#include "bf16_dot.cuh"
 
 namespace cp {
 
@@ -12,24 +13,6 @@ namespace cp {
 // neighbour order by one thread.
 constexpr int CAP_WARPS = 8;
 
-// acc + x . y over the 8 bf16 of each operand, element order lo, hi of each
-// 32-bit word in turn: fma.rn.f32.bf16 takes the bf16 operands as they are
-// (their product is exact in fp32) and rounds once, so each step equals
-// fmaf on the widened values and the sum is the same as widening first.
-__device__ __forceinline__ float dot8_bf16(const uint4 x, const uint4 y, float acc) {
-  asm("{\n\t.reg .b16 xl, xh, yl, yh;\n\t"
-      "mov.b32 {xl, xh}, %1;\n\tmov.b32 {yl, yh}, %5;\n\t"
-      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t"
-      "mov.b32 {xl, xh}, %2;\n\tmov.b32 {yl, yh}, %6;\n\t"
-      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t"
-      "mov.b32 {xl, xh}, %3;\n\tmov.b32 {yl, yh}, %7;\n\t"
-      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t"
-      "mov.b32 {xl, xh}, %4;\n\tmov.b32 {yl, yh}, %8;\n\t"
-      "fma.rn.f32.bf16 %0, xl, yl, %0;\n\tfma.rn.f32.bf16 %0, xh, yh, %0;\n\t}"
-      : "+f"(acc)
-      : "r"(x.x), "r"(x.y), "r"(x.z), "r"(x.w), "r"(y.x), "r"(y.y), "r"(y.z), "r"(y.w));
-  return acc;
-}
 template <typename T>
 __device__ __forceinline__ float row_dot(const T* a, const T* b, int D, int lane) {
   constexpr int V = Vec16<T>::n;

@@ -1,6 +1,7 @@
 // K0 (scene statistics, inverse feature norms), K1 (3D nearest neighbours and
 // scene diameter) and the min-max normalisers of Sec. 3.3.
 #include "common.cuh"
+#include "bf16_dot.cuh"
 
 namespace cp {
 
@@ -77,11 +78,18 @@ __global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ F,
   const T* f = F + row * D;
   constexpr int V = Vec16<T>::n;
   float acc = 0.0f;
-  for (int d = lane * V; d < D; d += 32 * V) {
-    float x[V];
-    Vec16<T>::load(f + d, x);
+  if constexpr (V == 8) {  // bf16: the same products and order, no widening
+    for (int d = lane * V; d < D; d += 32 * V) {
+      const uint4 x = __ldg(reinterpret_cast<const uint4*>(f + d));
+      acc = dot8_bf16(x, x, acc);
+    }
+  } else {
+    for (int d = lane * V; d < D; d += 32 * V) {
+      float x[V];
+      Vec16<T>::load(f + d, x);
 #pragma unroll
-    for (int i = 0; i < V; ++i) acc = fmaf(x[i], x[i], acc);
+      for (int i = 0; i < V; ++i) acc = fmaf(x[i], x[i], acc);
+    }
   }
   acc = warp_sum(acc);
   if (lane == 0) {
