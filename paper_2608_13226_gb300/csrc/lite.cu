@@ -288,6 +288,22 @@ __device__ __forceinline__ uint4 ld_row16(const __nv_bfloat16* row, int col, int
   return (row != nullptr && col < D) ? __ldg(reinterpret_cast<const uint4*>(row + col))
                                      : make_uint4(0u, 0u, 0u, 0u);
 }
+// ld_row16 as an asynchronous copy into shared memory (zeros where it gives
+// zeros: no bytes are read then, and src is only a valid placeholder)
+__device__ __forceinline__ void cp_row16(uint4* dst, const __nv_bfloat16* row, int col, int D,
+                                         const void* any) {
+  const bool ok = row != nullptr && col < D;
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d),
+               "l"(ok ? (const void*)(row + col) : any), "r"(ok ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+constexpr int LP_STAGES = 4;  // chunks of a warp in flight (diagonal tiles)
 __global__ void __launch_bounds__(32 * LP_WARPS) k_lite_proto_tc(
     const __nv_bfloat16* __restrict__ F_all, const float* __restrict__ inv_all,
     const float* __restrict__ pos_all, const int32_t* __restrict__ frame_all,
@@ -296,6 +312,8 @@ __global__ void __launch_bounds__(32 * LP_WARPS) k_lite_proto_tc(
     int D, int K, int32_t* __restrict__ proto, double* __restrict__ score) {
   __shared__ float s_dot[LP_MAXG][LP_MAXG + 1];
   __shared__ float s_part[LP_WARPS][16][17];
+  // diagonal tiles: each lane's two 16-byte pieces of a chunk, LP_STAGES deep
+  __shared__ __align__(16) uint4 s_stg[LP_WARPS][LP_STAGES][2][32];
   __shared__ float s_inv[LP_MAXG], s_v[LP_MAXG], s_x[LP_MAXG][3];
   __shared__ int s_mem[LP_MAXG], s_tau[LP_MAXG];
   __shared__ float s_sc[LP_WARPS];
@@ -338,8 +356,36 @@ __global__ void __launch_bounds__(32 * LP_WARPS) k_lite_proto_tc(
         const __nv_bfloat16* pb0 = rb0 < sz ? F + (size_t)s_mem[rb0] * D : nullptr;
         const __nv_bfloat16* pb1 = rb1 < sz ? F + (size_t)s_mem[rb1] * D : nullptr;
         float d0[4] = {0.f, 0.f, 0.f, 0.f}, d1[4] = {0.f, 0.f, 0.f, 0.f};
+        if (bi == bj) {
+          // the same chunks and MMAs as below, the rows brought in by
+          // asynchronous copies LP_STAGES chunks ahead (each lane reads
+          // back only its own copies)
+          const int nch = (D - 32 * w + 32 * LP_WARPS - 1) / (32 * LP_WARPS);
+          auto issue = [&](int i) {
+            const int col = 32 * w + 32 * LP_WARPS * i + 8 * tg;
+            cp_row16(&s_stg[w][i % LP_STAGES][0][lane], pa0, col, D, F);
+            cp_row16(&s_stg[w][i % LP_STAGES][1][lane], pa1, col, D, F);
+          };
+#pragma unroll
+          for (int i = 0; i < LP_STAGES - 1; ++i) {
+            if (i < nch) issue(i);
+            cp_commit();
+          }
+          for (int i = 0; i < nch; ++i) {
+            if (i + LP_STAGES - 1 < nch) issue(i + LP_STAGES - 1);
+            cp_commit();
+            cp_wait<LP_STAGES - 1>();  // chunk i has landed
+            const uint4 x0 = s_stg[w][i % LP_STAGES][0][lane];
+            const uint4 x1 = s_stg[w][i % LP_STAGES][1][lane];
+            mma_bf16_16816(d0, x0.x, x1.x, x0.y, x1.y, x0.x, x0.y);
+            mma_bf16_16816(d1, x0.x, x1.x, x0.y, x1.y, x1.x, x1.y);
+            mma_bf16_16816(d0, x0.z, x1.z, x0.w, x1.w, x0.z, x0.w);
+            mma_bf16_16816(d1, x0.z, x1.z, x0.w, x1.w, x1.z, x1.w);
+          }
+          cp_wait<0>();
+        }
 #pragma unroll 2
-        for (int c0 = 32 * w; c0 < D; c0 += 32 * LP_WARPS) {
+        for (int c0 = 32 * w; bi != bj && c0 < D; c0 += 32 * LP_WARPS) {
           const int col = c0 + 8 * tg;
           const uint4 x0 = ld_row16(pa0, col, D), x1 = ld_row16(pa1, col, D);
           uint4 y0 = x0, y1 = x1;  // bi == bj: B rows are A's
