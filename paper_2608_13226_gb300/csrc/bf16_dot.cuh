@@ -1,6 +1,8 @@
-// Dot products of bf16 rows with fp32 accumulation on the mixed-precision
-// FMA (fma.rn.f32.bf16): the bf16 operands enter the FMA as they are, with
-// no widening instructions.
+// bf16 rows: dot products with fp32 accumulation on the mixed-precision FMA
+// (fma.rn.f32.bf16: the bf16 operands enter the FMA as they are, with no
+// widening instructions), and 16-byte asynchronous copies of row pieces into
+// shared memory (cp.async), for loops that keep several pieces in flight
+// without holding them in registers.
 #pragma once
 #include <stdint.h>
 
@@ -24,4 +26,27 @@ __device__ __forceinline__ float dot8_bf16(const uint4 x, const uint4 y, float a
       : "r"(x.x), "r"(x.y), "r"(x.z), "r"(x.w), "r"(y.x), "r"(y.y), "r"(y.z), "r"(y.w));
   return acc;
 }
+// 16 bytes global -> shared, cached in L1 as well (rows that other warps of
+// the block read too)
+__device__ __forceinline__ void cp_async16_ca(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 16;" ::"r"(
+                   (uint32_t)__cvta_generic_to_shared(dst)),
+               "l"(src)
+               : "memory");
+}
+// 16 bytes global -> shared through L2 only; zeros, reading nothing, when
+// !ok (src must still be a valid address)
+__device__ __forceinline__ void cp_async16_zfill(void* dst, const void* src, bool ok) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(
+                   (uint32_t)__cvta_generic_to_shared(dst)),
+               "l"(src), "r"(ok ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// this thread's copies of all but the newest N committed groups have landed
+template <int N>
+__device__ __forceinline__ void cp_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 }  // namespace cp

@@ -1,6 +1,7 @@
 // K6-K8: CoverPrune-Lite (Sec. 4.1, Eqs. lite_group, lite_select; Sec. 4.2,
 // Eqs. blk_plan, blk_ot).
 #include "common.cuh"
+#include "bf16_dot.cuh"
 
 namespace cp {
 
@@ -289,19 +290,11 @@ __device__ __forceinline__ uint4 ld_row16(const __nv_bfloat16* row, int col, int
                                      : make_uint4(0u, 0u, 0u, 0u);
 }
 // ld_row16 as an asynchronous copy into shared memory (zeros where it gives
-// zeros: no bytes are read then, and src is only a valid placeholder)
+// zeros: no bytes are read then, and F itself stands in as the source)
 __device__ __forceinline__ void cp_row16(uint4* dst, const __nv_bfloat16* row, int col, int D,
                                          const void* any) {
   const bool ok = row != nullptr && col < D;
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d),
-               "l"(ok ? (const void*)(row + col) : any), "r"(ok ? 16 : 0)
-               : "memory");
-}
-__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+  cp_async16_zfill(dst, ok ? (const void*)(row + col) : any, ok);
 }
 constexpr int LP_STAGES = 4;  // chunks of a warp in flight (diagonal tiles)
 __global__ void __launch_bounds__(32 * LP_WARPS) k_lite_proto_tc(
