@@ -465,13 +465,16 @@ def run_ours(args, rank, world, local_rank, raw):
     e2e_ms = max_over_ranks(a.elapsed_time(b_) / n_e2e)
     h2d = feats_pin.numel() * 2 + pos_pin.numel() * 4 + fr_pin.numel() * 4
     d2h = kept_pin.numel() * 8 + obj_pin.numel() * 8
-    # the upload alone, for context (host-to-device bandwidth of this machine)
-    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    c0.record(stream)
-    inputs[0][0].copy_(feats_pin, non_blocking=True)
-    c1.record(stream)
-    torch.cuda.synchronize()
-    h2d_gbs = feats_pin.numel() * 2 / (c0.elapsed_time(c1) / 1000.0) / 1e9
+    # the upload alone, for context (host-to-device bandwidth of this machine;
+    # the best of three copies)
+    h2d_gbs = 0.0
+    for _ in range(3):
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0.record(stream)
+        inputs[0][0].copy_(feats_pin, non_blocking=True)
+        c1.record(stream)
+        torch.cuda.synchronize()
+        h2d_gbs = max(h2d_gbs, feats_pin.numel() * 2 / (c0.elapsed_time(c1) / 1000.0) / 1e9)
     e2e = {"value": B * world / (e2e_ms / 1000.0), "unit": "scenes/s",
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 3),
            "steps": n_e2e, "h2d_GBps": round(h2d_gbs, 1),
