@@ -470,6 +470,7 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_local(
   uint32_t* chosen = reinterpret_cast<uint32_t*>(ub + N);  // [nwords]
   uint32_t* fresh = chosen + nwords;                       // [nwords]
   __shared__ unsigned long long s_wkey[LZ_WARPS];          // each warp's best key
+  __shared__ unsigned long long s_wkey2[LZ_WARPS];         // ... and its second best
   __shared__ int s_wfr[LZ_WARPS];                          // ... and whether it is exact
   __shared__ int s_pick, s_bad;
   unsigned long long my_evals = 0ull, my_rounds = 0ull, my_bytes = 0ull;
@@ -505,16 +506,30 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_local(
     const int t = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
     return key != 0ull && ((fresh[t >> 5] >> (t & 31)) & 1u);
   };
-  auto rescan = [&]() {
-    unsigned long long best = 0ull;
+  auto rescan = [&]() {  // the warp's best and second-best keys
+    unsigned long long best = 0ull, second = 0ull;
     for (int t = w + LZ_WARPS * lane; t < N; t += LZ_WARPS * 32)
       if (!(chosen[t >> 5] & (1u << (t & 31)))) {
         const unsigned long long key = gain_key(ub[t], t);
-        best = key > best ? key : best;
+        if (key > best) {
+          second = best;
+          best = key;
+        } else if (key > second) {
+          second = key;
+        }
       }
-    best = warp_max_u64(best);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {  // merge the lanes' top two
+      const unsigned long long ob = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+      const unsigned long long os = __shfl_xor_sync(0xFFFFFFFFu, second, o);
+      const unsigned long long lo = best < ob ? best : ob;
+      best = best > ob ? best : ob;
+      const unsigned long long s2 = second > os ? second : os;
+      second = lo > s2 ? lo : s2;
+    }
     if (lane == 0) {
       s_wkey[w] = best;
+      s_wkey2[w] = second;
       s_wfr[w] = is_fresh(best);
     }
   };
@@ -540,12 +555,23 @@ __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_local(
       if (G == 0ull) break;  // no candidate left (never for K <= N)
       if (!mine_fresh && mine > BF) {  // this slice's best might still win
         const int t = (int)(0xFFFFFFFFu - (uint32_t)(mine & 0xFFFFFFFFull));
+        // so may its second best when stale and above the largest exact
+        // key: evaluated in the same round (any stale candidate may be)
+        const unsigned long long k2 = s_wkey2[w];
+        const int t2 = (k2 > BF && !is_fresh(k2)) ? (int)(0xFFFFFFFFu - (uint32_t)(k2 & 0xFFFFFFFFull))
+                                                  : -1;
         const float gt = gain_of(t);
+        const float gt2 = t2 >= 0 ? gain_of(t2) : 0.0f;
         ++my_evals;
         if (lane == 0) {
           ub[t] = gt;
           atomicOr(&fresh[t >> 5], 1u << (t & 31));
+          if (t2 >= 0) {
+            ub[t2] = gt2;
+            atomicOr(&fresh[t2 >> 5], 1u << (t2 & 31));
+          }
         }
+        if (t2 >= 0) ++my_evals;
         __syncwarp();
         rescan();
       }
