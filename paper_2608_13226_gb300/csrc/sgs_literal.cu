@@ -18,11 +18,11 @@
 //
 // The path is HBM-bound: each iteration reads the l selected rows of the
 // dense cost twice (rows, then columns), the score reads every candidate's
-// row once.  One launch per phase covers all B scenes: rows a warp per
-// source row, columns a thread per target column (the l source indices and
-// potentials staged in shared memory, the cost read coalesced along the
-// row; a block spreads 32 columns over 8 groups of source rows), scores a
-// warp per candidate.  Each step's winner is the smallest
+// row once.  One launch per phase covers all B scenes: columns a thread per
+// target column (the l source indices and potentials staged in shared
+// memory, the cost read coalesced along the row; a block spreads 32 columns
+// over 8 groups of source rows), rows a block per source row, scores a warp
+// per candidate; every thread keeps eight loads in flight.  Each step's winner is the smallest
 // (score bits, index) key, reduced with one 64-bit atomicMin per block into
 // that step's slot (initialised to all ones), so no separate argmin pass
 // runs; non-negative floats order like their bit patterns, and every score
@@ -73,21 +73,42 @@ __device__ __forceinline__ int key_index(unsigned long long k) {
 }
 
 // Row potentials of the l sources: f_i = eps log u - eps LSE_j((g_j - C_ij) / eps).
+// One block per source row: thread x takes the columns x, x + 256, ...,
+// eight loads in flight before their terms are added in column order; the
+// threads' partial log-sum-exps merge in a fixed order (warps by butterfly,
+// then the 8 warps in order).
 __global__ void __launch_bounds__(LIT_THREADS) k_lit_rows(
     const float* __restrict__ C, int64_t ldc, int N, int K, int l,
     const unsigned long long* __restrict__ keys, const float* __restrict__ gpot, float eps,
     float inv_eps, float log_u, float* __restrict__ fpot) {
-  const int b = blockIdx.y;
-  const int i = blockIdx.x * (LIT_THREADS / 32) + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (i >= l) return;
+  __shared__ float s_m[LIT_THREADS / 32], s_s[LIT_THREADS / 32];
+  const int b = blockIdx.y, i = blockIdx.x;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int s = key_index(keys[(size_t)b * K + i]);
   const float* row = C + ((size_t)b * N + s) * ldc;
   const float* g = gpot + (size_t)b * N;
   Lse a{-INFINITY, 0.0f};
-  for (int j = lane; j < N; j += 32) lse_add(a, (__ldg(g + j) - __ldg(row + j)) * inv_eps);
+  for (int j0 = threadIdx.x; j0 < N; j0 += 8 * LIT_THREADS) {
+    float x[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int j = j0 + u * LIT_THREADS;
+      x[u] = j < N ? (__ldg(g + j) - __ldg(row + j)) * inv_eps : -INFINITY;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) lse_add(a, x[u]);
+  }
   a = warp_lse(a);
-  if (lane == 0) fpot[(size_t)b * K + i] = eps * (log_u - lse_value(a));
+  if (lane == 0) {
+    s_m[w] = a.m;
+    s_s[w] = a.s;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    Lse t{s_m[0], s_s[0]};
+    for (int q = 1; q < LIT_THREADS / 32; ++q) t = lse_merge(t, Lse{s_m[q], s_s[q]});
+    fpot[(size_t)b * K + i] = eps * (log_u - lse_value(t));
+  }
 }
 
 // Per target column j, LSE_i((f_i - C(s_i, j)) / eps) over the l sources.
@@ -124,8 +145,17 @@ __global__ void __launch_bounds__(LC_COLS * LC_GROUPS) k_lit_cols(
     }
     __syncthreads();
     if (j < N)
-      for (int ii = ty; ii < n; ii += LC_GROUPS)
-        lse_add(a, (s_f[ii] - __ldg(Cb + (size_t)s_idx[ii] * ldc + j)) * inv_eps);
+      for (int i1 = ty; i1 < n; i1 += 8 * LC_GROUPS) {  // eight loads in flight
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int ii = i1 + u * LC_GROUPS;
+          x[u] = ii < n ? (s_f[ii] - __ldg(Cb + (size_t)s_idx[ii] * ldc + j)) * inv_eps
+                        : -INFINITY;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) lse_add(a, x[u]);
+      }
   }
   s_m[ty][tx] = a.m;
   s_s[ty][tx] = a.s;
@@ -272,7 +302,7 @@ int launch_sgs_literal(const float* cost, int64_t ldc, const int32_t* nbr, const
   const dim3 gscore((unsigned)((N + LIT_THREADS / 32 - 1) / (LIT_THREADS / 32)), (unsigned)B);
   for (int l = 0; l < k; ++l) {
     if (l > 0) {
-      const dim3 grows((unsigned)((l + LIT_THREADS / 32 - 1) / (LIT_THREADS / 32)), (unsigned)B);
+      const dim3 grows((unsigned)l, (unsigned)B);
       for (int it = 0; it < P.sot_iters; ++it) {
         k_lit_rows<<<grows, LIT_THREADS, 0, s>>>(cost, ldc, n, k, l, keys, gpot, eps, inv_eps,
                                                  log_u, fpot);
