@@ -21,7 +21,7 @@
 // row once.  One launch per phase covers all B scenes: columns a thread per
 // target column (the l source indices and potentials staged in shared
 // memory, the cost read coalesced along the row; a block spreads 32 columns
-// over 8 groups of source rows), rows a block per source row, scores a warp
+// over 16 groups of source rows), rows a block per source row, scores a warp
 // per candidate; every thread keeps eight loads in flight.  Each step's winner is the smallest
 // (score bits, index) key, reduced with one 64-bit atomicMin per block into
 // that step's slot (initialised to all ones), so no separate argmin pass
@@ -112,13 +112,13 @@ __global__ void __launch_bounds__(LIT_THREADS) k_lit_rows(
 }
 
 // Per target column j, LSE_i((f_i - C(s_i, j)) / eps) over the l sources.
-// A block takes 32 columns (threadIdx.x) and splits the sources over 8 row
-// groups (threadIdx.y: i = y, y + 8, ...), each warp reading 128
-// contiguous bytes of a source row; the 8 partial log-sum-exps of a column
+// A block takes 32 columns (threadIdx.x) and splits the sources over 16 row
+// groups (threadIdx.y: i = y, y + 16, ...), each warp reading 128
+// contiguous bytes of a source row; the 16 partial log-sum-exps of a column
 // merge in a fixed order.  RESID = false: the column potential g_j (the
 // capacity cap).  RESID = true: the residual r_j = max(v_j - exp(g_j / eps +
 // LSE), 0), and block 0 marks the previous step's pick as selected.
-constexpr int LC_COLS = 32, LC_GROUPS = 8, LC_CHUNK = 256;
+constexpr int LC_COLS = 32, LC_GROUPS = 16, LC_CHUNK = 256;
 template <bool RESID>
 __global__ void __launch_bounds__(LC_COLS * LC_GROUPS) k_lit_cols(
     const float* __restrict__ C, int64_t ldc, int N, int K, int l,
