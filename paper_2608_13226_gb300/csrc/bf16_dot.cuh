@@ -26,14 +26,6 @@ __device__ __forceinline__ float dot8_bf16(const uint4 x, const uint4 y, float a
       : "r"(x.x), "r"(x.y), "r"(x.z), "r"(x.w), "r"(y.x), "r"(y.y), "r"(y.z), "r"(y.w));
   return acc;
 }
-// 16 bytes global -> shared, cached in L1 as well (rows that other warps of
-// the block read too)
-__device__ __forceinline__ void cp_async16_ca(void* dst, const void* src) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 16;" ::"r"(
-                   (uint32_t)__cvta_generic_to_shared(dst)),
-               "l"(src)
-               : "memory");
-}
 // 16 bytes global -> shared through L2 only; zeros, reading nothing, when
 // !ok (src must still be a valid address)
 __device__ __forceinline__ void cp_async16_zfill(void* dst, const void* src, bool ok) {

@@ -350,9 +350,9 @@ __global__ void __launch_bounds__(32 * LP_WARPS) k_lite_proto_tc(
         const __nv_bfloat16* pb1 = rb1 < sz ? F + (size_t)s_mem[rb1] * D : nullptr;
         float d0[4] = {0.f, 0.f, 0.f, 0.f}, d1[4] = {0.f, 0.f, 0.f, 0.f};
         if (bi == bj) {
-          // the same chunks and MMAs as below, the rows brought in by
-          // asynchronous copies LP_STAGES chunks ahead (each lane reads
-          // back only its own copies)
+          // diagonal tile (B rows are A's): the same chunks and MMAs as the
+          // loop below, the rows brought in by asynchronous copies
+          // LP_STAGES chunks ahead (each lane reads back only its own copies)
           const int nch = (D - 32 * w + 32 * LP_WARPS - 1) / (32 * LP_WARPS);
           auto issue = [&](int i) {
             const int col = 32 * w + 32 * LP_WARPS * i + 8 * tg;
@@ -377,15 +377,12 @@ __global__ void __launch_bounds__(32 * LP_WARPS) k_lite_proto_tc(
           }
           cp_wait<0>();
         }
+        // off-diagonal tiles (groups of more than 16): A and B rows loaded
 #pragma unroll 2
         for (int c0 = 32 * w; bi != bj && c0 < D; c0 += 32 * LP_WARPS) {
           const int col = c0 + 8 * tg;
           const uint4 x0 = ld_row16(pa0, col, D), x1 = ld_row16(pa1, col, D);
-          uint4 y0 = x0, y1 = x1;  // bi == bj: B rows are A's
-          if (bi != bj) {
-            y0 = ld_row16(pb0, col, D);
-            y1 = ld_row16(pb1, col, D);
-          }
+          const uint4 y0 = ld_row16(pb0, col, D), y1 = ld_row16(pb1, col, D);
           // k16 step over columns 8 tg + {0..3} of every lane, then + {4..7}
           mma_bf16_16816(d0, x0.x, x1.x, x0.y, x1.y, y0.x, y0.y);
           mma_bf16_16816(d1, x0.x, x1.x, x0.y, x1.y, y1.x, y1.y);
