@@ -567,7 +567,7 @@ def _lite_check(orc, s, K, prm, dtype):
 
 
 @pytest.mark.parametrize("n_cap", [3, 8, 12])
-@pytest.mark.parametrize("N,D,seed", [(1001, 512, 6), (4100, 1280, 7)])
+@pytest.mark.parametrize("N,D,seed", [(1001, 512, 6), (4100, 1280, 7), (777, 200, 8)])
 def test_capacity_from_features(orc, n_cap, N, D, seed):
     """The capacity computed from the bf16 features (Lite, and cost calls
     without the cost) at ragged N and several neighbour counts, against the
@@ -616,6 +616,17 @@ def test_lite_bounded_normaliser(orc, name, N, D, K):
     s = scene(name, 2, N=N, D=D)
     near = _lite_check(orc, s, K, cp.Params(norm_mode=1), s["dtype"])
     print(f"lite bounded {name}: near-tie prototype differences {near}/{K}")
+
+
+@pytest.mark.parametrize("K", [12, 25, 90])
+def test_lite_group_sizes_ragged_width(orc, K):
+    """Groups of ~83 members (the FMA path past 64), ~40 (several tensor-core
+    tiles a group, off-diagonal tiles included) and ~11 (one diagonal tile
+    fed by asynchronous copies), on a feature width that is not a multiple
+    of any chunk (D = 200: the last 32-column chunk is a quarter full)."""
+    s = scene("long_video", 3, N=1000, D=200)
+    _lite_check(orc, s, K, cp.Params(), "bf16")
+    _lite_check(orc, s, K, cp.Params(norm_mode=1), "bf16")
 
 
 def test_lite_edges(orc):
