@@ -141,6 +141,16 @@ typedef enum {
  *                                   and temporal normalisers are the same in
  *                                   both.  The two agree whenever the scene
  *                                   holds a pair with cos = -1.
+ *   inputs_done                     not a method parameter: a cudaEvent_t
+ *                                   (passed as void*) or NULL.  When given,
+ *                                   the call records it on its stream once it
+ *                                   has read the last of feats, pos and frame;
+ *                                   work ordered after that event may
+ *                                   overwrite them (a serving loop's next
+ *                                   upload, say).  coverprune_select records
+ *                                   it before its greedy selection, the other
+ *                                   calls on return.  The caller owns the
+ *                                   event (default NULL).
  */
 typedef struct {
   uint32_t struct_size; /* = sizeof(cp_params); set by cp_default_params */
@@ -157,6 +167,7 @@ typedef struct {
   int32_t norm_mode;
   float sot_eps;
   int32_t sot_iters;
+  void* inputs_done;
 } cp_params;
 
 /* Fills *p with the defaults listed above.  Host only; p must not be NULL. */

@@ -49,7 +49,8 @@ class _CpParams(C.Structure):
                 ("n_cap", C.c_int32), ("g", C.c_int32), ("capacity_mode", C.c_int32),
                 ("voxel_m", C.c_float), ("m0", C.c_float), ("timeout_ms", C.c_float),
                 ("sgs_mode", C.c_int32), ("norm_mode", C.c_int32),
-                ("sot_eps", C.c_float), ("sot_iters", C.c_int32)]
+                ("sot_eps", C.c_float), ("sot_iters", C.c_int32),
+                ("inputs_done", C.c_void_p)]
 
 
 class _CallStats(C.Structure):
@@ -78,12 +79,21 @@ class Params:
     norm_mode: int = 0
     sot_eps: float = 0.05
     sot_iters: int = 20
+    # not a method parameter: a torch.cuda.Event the call records once it has
+    # read the last of its inputs (cp_params.inputs_done), or None
+    inputs_done: object = None
 
     def _c(self) -> _CpParams:
         p = _CpParams()
         _lib().cp_default_params(C.byref(p))
         for f in fields(self):
-            setattr(p, f.name, getattr(self, f.name))
+            if f.name == "inputs_done":
+                ev = self.inputs_done
+                if ev is not None and not ev.cuda_event:
+                    ev.record()  # torch creates its CUDA event on first record
+                p.inputs_done = None if ev is None else C.c_void_p(ev.cuda_event)
+            else:
+                setattr(p, f.name, getattr(self, f.name))
         return p
 
 

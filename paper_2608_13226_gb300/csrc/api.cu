@@ -360,6 +360,13 @@ static int check_ws(int op, int64_t B, int64_t N, int64_t D, int64_t K, int dtyp
   return CP_OK;
 }
 
+// Records the caller's inputs_done event (cp_params) on the call's stream.
+static int record_inputs_done(const cp_params* p, cudaStream_t s) {
+  if (!p->inputs_done) return CP_OK;
+  return cuda_status(cudaEventRecord(static_cast<cudaEvent_t>(p->inputs_done), s),
+                     "inputs_done event");
+}
+
 }  // namespace cp
 
 using namespace cp;
@@ -383,6 +390,7 @@ void cp_default_params(cp_params* p) {
   p->norm_mode = 0;
   p->sot_eps = 0.05f;
   p->sot_iters = 20;
+  p->inputs_done = nullptr;
 }
 
 int64_t coverprune_budget(double R, int64_t N) {
@@ -489,7 +497,7 @@ int coverprune_cost(const void* feats, int dtype, const float* pos, const int32_
       CP_TRY(launch_cost(feats, dtype, at<float>(ws, pl.inv), at<float4>(ws, pl.tok), pos, frame,
                          nm, d, B, N, D, cost, N, s));
   }
-  return CP_OK;
+  return record_inputs_done(p, s);
 }
 
 int coverprune_select(const void* feats, int dtype, const float* pos, const int32_t* frame,
@@ -558,6 +566,8 @@ int coverprune_select(const void* feats, int dtype, const float* pos, const int3
       CP_TRY(launch_cost(feats, dtype, inv, at<float4>(ws, pl.tok), pos, frame, nm, d, B, N, D, C,
                          pl.ldc, s));
   }
+  // the greedy selection reads none of feats, pos, frame
+  CP_TRY(record_inputs_done(p, s));
   int32_t* order32 = at<int32_t>(ws, pl.order32);
   {
     Stage st(CP_STAGE_SGS, s);
@@ -616,6 +626,7 @@ int coverprune_lite_select(const void* feats, int dtype, const float* pos, const
     CP_TRY(launch_lite_proto(feats, dtype, inv, pos, frame, nm, v, perm, gs, d, B, N, D, K, proto,
                              at<double>(ws, pl.score), objective, s));
   }
+  CP_TRY(record_inputs_done(p, s));
   Stage st(CP_STAGE_OUTPUT, s);
   CP_TRY(launch_sort_kept(proto, B, K, kept, nullptr, s));
   return CP_OK;

@@ -517,6 +517,30 @@ def test_sgs_local_duplicates_equal_full_sweep():
             assert torch.equal(lazy[k], full[k]), (g, k)
 
 
+def test_inputs_done_event_allows_overwriting_inputs():
+    """cp_params.inputs_done is recorded once a call has read its inputs:
+    zeroing them on another stream right after that event (while the greedy
+    selection still runs) leaves every result as it was."""
+    s = scene("short_clip", 0, N=2000, D=256)
+    f, pos, fr = to_dev(s)
+    side = torch.cuda.Stream()
+    for call in ("select", "lite"):
+        fn = cp.coverprune_select if call == "select" else cp.coverprune_lite_select
+        ref = fn(f, pos, fr, 300)
+        f2, pos2, fr2 = f.clone(), pos.clone(), fr.clone()
+        ev = torch.cuda.Event()
+        r = fn(f2, pos2, fr2, 300, cp.Params(inputs_done=ev))
+        side.wait_event(ev)
+        with torch.cuda.stream(side):
+            f2.zero_()
+            pos2.zero_()
+            fr2.zero_()
+        torch.cuda.synchronize()
+        assert ev.query()
+        assert torch.equal(r["kept"], ref["kept"]), call
+        assert torch.equal(r["objective"], ref["objective"]), call
+
+
 def test_sgs_small_edges():
     for N in (1, 2, 3):
         f = torch.randn(N, 8, device="cuda").to(torch.bfloat16)
