@@ -454,7 +454,8 @@ __global__ void __launch_bounds__(1024) k_rev_build(const int32_t* __restrict__ 
 // and so its rounded sum, are unchanged.  A round reads every warp's best key
 // and whether it is exact: if the block's largest is exact it is the winner,
 // otherwise each warp whose best is stale and above the largest exact one
-// re-evaluates it (one warp a row, local_row_gain) and rescans its slice.
+// re-evaluates it (one warp a row, local_row_gain), and its second best too
+// when that one is stale and above it as well, then rescans its slice.
 // Step 0 evaluates every candidate; no inter-block synchronisation.
 __global__ void __launch_bounds__(LZ_THREADS, 1) k_sgs_local(
     const float* __restrict__ slab, const int32_t* __restrict__ nbr,
