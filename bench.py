@@ -669,6 +669,35 @@ def measure_configs(args, dev, stream, sync, max_over_ranks, feats, pos, fr, wor
         if st != cp.CP_OK:
             raise RuntimeError(f"device status after {what}: {cp.status_string(st)}")
 
+    def two_in_flight(K, prm_s, n):
+        """ms per call with two batches in flight: calls alternate between two
+        streams, each with its own workspace, so one call's greedy selection
+        (which leaves SMs idle: a block a scene for local SGS, 128 of 152 SMs
+        for the dense one) overlaps the next call's front end.  CUDA events:
+        from a start both streams wait on to the later of their two ends."""
+        streams = [torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)]
+        calls = [select_call(feats, pos, fr, K, prm_s) for _ in range(2)]
+
+        def run(i):
+            with torch.cuda.stream(streams[i % 2]):
+                calls[i % 2][0]()
+        for i in range(4):  # warm-up
+            run(i)
+        sync()
+        t0 = torch.cuda.Event(enable_timing=True)
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        t0.record(streams[0])
+        streams[1].wait_event(t0)
+        for i in range(n):
+            run(i)
+        for k in range(2):
+            ends[k].record(streams[k])
+        sync()
+        ms = max(t0.elapsed_time(e) for e in ends) / n
+        for _, w in calls:
+            check(w, "two calls in flight")
+        return ms
+
     # ---- single scenes
     for name in ("tiny", "short_clip", "long_video", "lite_long"):
         if name == "long_video":
@@ -743,6 +772,12 @@ def measure_configs(args, dev, stream, sync, max_over_ranks, feats, pos, fr, wor
                                "gain_evaluations_per_step": gst["gain_evaluations"]},
                               **sgs_numbers(stages, K, None, hbm))
                 del ws
+            two = {}
+            for key, pl in (("select", prm), ("select_local_g64", cp.Params(g=LOCAL_G)),
+                            ("select_local_g64_bounded", cp.Params(g=LOCAL_G, norm_mode=1))):
+                ms = max_over_ranks(two_in_flight(K, pl, max(8, args.steps)))
+                two[key] = {"scenes_per_s": B * world / (ms / 1000.0), "ms_per_step": round(ms, 3)}
+            e["two_batches_in_flight"] = two
         floor_ms = B * N * D * 2 / (hbm * 1e9) * 1e3  # one read of the features
         for key, pr in (("lite", prm), ("lite_bounded", bounded)):
             call, ws = lite_call(feats, pos, fr, K, pr)
@@ -757,7 +792,9 @@ def measure_configs(args, dev, stream, sync, max_over_ranks, feats, pos, fr, wor
     out["batch32_sweep"] = sweep
     out["notes"] = ("bounded = the bounded feature normaliser (d_f / 2), no all-pairs Gram; "
                     "latency = one call timed alone (median of 5 after 2 warm-ups); "
-                    "batch numbers: CUDA events over back-to-back calls on resident inputs")
+                    "batch numbers: CUDA events over back-to-back calls on resident inputs; "
+                    "two_batches_in_flight: the same calls alternating between two streams "
+                    "with a workspace each (a serving loop with two batches in flight)")
     return out
 
 
